@@ -1,0 +1,108 @@
+"""Brute-force and first-principles checks used to pin the oracle.
+
+Nothing here calls the oracle or the CUDA library; every function is written
+from a definition in the paper that is more primitive than the one under test:
+  * the materialisation rule of Section III-A (local copy 0, peer-only
+    min{w, f}, none w) for the objectives,
+  * "parent-closed subset within the budget" (Eq. 8) enumerated exhaustively
+    for the DP and for the joint optimum.
+"""
+from __future__ import annotations
+
+import itertools
+
+import numpy as np
+
+
+def materialisation_saving(inst, placement) -> int:
+    """Savings over all-recompute, straight from Section III-A.
+
+    Requester m needing chunk b pays 0 if it holds b; otherwise the cheapest of
+    recomputation w_m(b) and fetching from any holder; w_m(b) with no holder.
+    Source-dependent costs (mode 1) use f_{m<-h}(b) = transfer[h][m][b]."""
+    W, n = inst.W, inst.n
+    pl = np.asarray(placement, bool)
+    total = 0
+    for b in range(n):
+        holders = [h for h in range(W) if pl[h, b]]
+        for m in range(W):
+            w = int(inst.recompute[m, b])
+            if pl[m, b]:
+                cost = 0
+            elif holders:
+                if inst.mode == 0:
+                    fetch = int(inst.transfer[m, b])
+                else:
+                    fetch = min(int(inst.transfer[h, m, b]) for h in holders)
+                cost = min(w, fetch)
+            else:
+                cost = w
+            total += int(inst.demand[m, b]) * (w - cost)
+    return total
+
+
+def parent_closed_masks(parent, weight, k):
+    """All parent-closed subsets of total weight <= k, as an (N, n) bool array."""
+    parent = np.asarray(parent)
+    n = parent.shape[0]
+    masks = np.arange(1 << n, dtype=np.int64)
+    bits = ((masks[:, None] >> np.arange(n)[None, :]) & 1).astype(bool)
+    ok = np.ones(masks.shape[0], bool)
+    for v in range(n):
+        p = parent[v]
+        if p >= 0:
+            ok &= ~bits[:, v] | bits[:, p]
+    wsum = bits.astype(np.int64) @ np.asarray(weight, np.int64)
+    ok &= wsum <= k
+    return bits[ok]
+
+
+def preorder_positions(parent):
+    """Preorder with roots then children in ascending node id (plain recursion)."""
+    parent = list(int(p) for p in parent)
+    n = len(parent)
+    kids = {u: [] for u in range(-1, n)}
+    for v in range(n):
+        kids[parent[v]].append(v)
+    order = []
+
+    def visit(u):
+        order.append(u)
+        for c in sorted(kids[u]):
+            visit(c)
+
+    for r in sorted(kids[-1]):
+        visit(r)
+    return order
+
+
+def best_parent_closed(parent, weight, profit, k):
+    """Maximum-profit parent-closed set of weight <= k, by enumeration.
+
+    Among optimal sets returns the lexicographically smallest 0/1 indicator
+    taken in preorder (0 before 1 at the earliest differing position)."""
+    sets = parent_closed_masks(parent, weight, k)
+    vals = sets.astype(np.int64) @ np.asarray(profit, np.int64)
+    best = vals.max()
+    opt = sets[vals == best]
+    order = preorder_positions(parent)
+    keys = [tuple(int(row[v]) for v in order) for row in opt]
+    i = min(range(len(keys)), key=lambda t: keys[t])
+    return int(best), opt[i].astype(np.uint8)
+
+
+def joint_optimum(inst) -> int:
+    """max over all feasible joint placements (Eq. 8) of the Section III-A saving."""
+    per = [parent_closed_masks(inst.parent, inst.weight, int(inst.budget[m])) for m in range(inst.W)]
+    best = 0
+    for combo in itertools.product(*[range(len(p)) for p in per]):
+        pl = np.stack([per[m][combo[m]] for m in range(inst.W)])
+        best = max(best, materialisation_saving(inst, pl))
+    return best
+
+
+def is_parent_closed(parent, chosen) -> bool:
+    parent = np.asarray(parent)
+    ch = np.asarray(chosen, bool)
+    has_p = parent >= 0
+    return bool(np.all(~ch[has_p] | ch[parent[has_p]]))

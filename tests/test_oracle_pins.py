@@ -1,0 +1,322 @@
+"""Pins of the CPU oracle against what the paper and mathematics fix.
+
+Each test names the passage it checks.  None of them retypes the oracle's own
+formula: they compare against exhaustive enumeration, against the more
+primitive materialisation rule of Section III-A, against closed forms
+(Theorem 2's spider) or against theorems (Lemma 1, Prop. 1, Theorem 3).
+"""
+import numpy as np
+import pytest
+
+from paper_2608_01655_gb300 import workloads as wl
+from tests import bruteforce as bf
+
+
+def _prob(oracle, inst):
+    return oracle.Problem.from_instance(inst)
+
+
+# ---------------------------------------------------------------- preorder ---
+def test_preorder_definition(oracle_lib):
+    """Section IV-A: preorder numbering and next(i) = first position after subtree."""
+    rng = np.random.default_rng(1)
+    for trial in range(30):
+        inst = wl.random_small(rng, int(rng.integers(1, 40)), 1, 0)
+        order, nxt = oracle_lib.preorder(inst.parent)
+        assert list(order) == bf.preorder_positions(inst.parent)
+        pos = np.empty(inst.n, int)
+        pos[order] = np.arange(inst.n)
+        # subtree of order[i] is exactly positions [i, next(i))
+        for i, v in enumerate(order):
+            sub = set()
+            stack = [v]
+            while stack:
+                u = stack.pop()
+                sub.add(u)
+                stack.extend(np.nonzero(inst.parent == u)[0].tolist())
+            assert sorted(pos[list(sub)]) == list(range(i, nxt[i]))
+
+
+def test_preorder_rejects_cycles(oracle_lib):
+    with pytest.raises(ValueError):
+        oracle_lib.preorder(np.array([1, 0, -1], np.int32))
+    with pytest.raises(ValueError):
+        oracle_lib.preorder(np.array([0], np.int32))
+    with pytest.raises(ValueError):
+        oracle_lib.preorder(np.array([5, -1], np.int32))
+
+
+# ------------------------------------------------------------- rooted DP ---
+@pytest.mark.parametrize("w_max", [1, 4])
+@pytest.mark.parametrize("variant", [0, 1])
+def test_rooted_dp_vs_bruteforce(oracle_lib, w_max, variant):
+    """Eq. 9 / Theorem 1: optimum over all parent-closed sets of weight <= k,
+    and the returned set is the lexicographically smallest preorder indicator
+    among optima (take only on a strict improvement)."""
+    rng = np.random.default_rng(10 + w_max + 7 * variant)
+    for trial in range(60):
+        n = int(rng.integers(1, 15))
+        inst = wl.random_small(rng, n, 1, 0, w_max=w_max)
+        # small profit range -> many ties; some zeros and a few negatives
+        profit = rng.integers(-2, 6, size=n).astype(np.int64)
+        if trial % 3 == 0:
+            profit = np.maximum(profit, 0)
+        k = int(rng.integers(0, n * w_max + 2))
+        best, chosen = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, k, variant)
+        bbest, bset = bf.best_parent_closed(inst.parent, inst.weight, profit, k)
+        assert best == bbest
+        np.testing.assert_array_equal(chosen, bset)
+
+
+def test_rooted_dp_variants_agree_on_configs(oracle_lib):
+    """The full-table and freed-row variants of Eq. 9 agree on real-sized trees."""
+    rng = np.random.default_rng(5)
+    for cfg in (0, 1):
+        inst = wl.make(cfg)
+        profit = rng.integers(0, 1000, size=inst.n).astype(np.int64)
+        profit[rng.random(inst.n) < 0.5] = 0
+        a = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, 300, 0)
+        b = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, 300, 1)
+        assert a[0] == b[0]
+        np.testing.assert_array_equal(a[1], b[1])
+
+
+def test_rooted_dp_special_cases(oracle_lib):
+    rng = np.random.default_rng(3)
+    # star forest of unit-weight roots: top-k profits; ties go to the later
+    # preorder position because skipping is preferred at the earliest one
+    n = 50
+    parent = np.full(n, -1, np.int32)
+    profit = rng.integers(0, 20, size=n).astype(np.int64)
+    for k in (0, 1, 7, 49, 50, 80):
+        best, ch = oracle_lib.rooted_dp(parent, np.ones(n, np.int32), profit, k)
+        top = sorted(range(n), key=lambda v: (-profit[v], -v))[:k]
+        top = [v for v in top if profit[v] > 0]
+        assert best == profit[top].sum()
+        assert set(np.nonzero(ch)[0]) == set(top)
+    # a single chain with non-negative profits: the first min(k, n) nodes,
+    # stopping after the last positive one
+    parent = np.arange(-1, n - 1, dtype=np.int32)
+    for k in (0, 3, 20, 60):
+        best, ch = oracle_lib.rooted_dp(parent, np.ones(n, np.int32), profit, k)
+        m = min(k, n)
+        assert best == profit[:m].sum()
+        pos = np.nonzero(profit[:m] > 0)[0]
+        last = pos[-1] + 1 if pos.size else 0
+        np.testing.assert_array_equal(ch, (np.arange(n) < last).astype(np.uint8))
+    # unlimited budget: exactly the nodes whose subtree holds a positive profit
+    inst = wl.random_small(rng, 200, 1, 0, w_max=3)
+    profit = rng.integers(0, 3, size=200).astype(np.int64) * (rng.random(200) < 0.1)
+    best, ch = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, int(inst.weight.sum()))
+    need = profit > 0
+    for v in range(200):
+        if profit[v] > 0:
+            u = inst.parent[v]
+            while u >= 0:
+                need[u] = True
+                u = inst.parent[u]
+    np.testing.assert_array_equal(ch.astype(bool), need)
+    assert best == profit.sum()
+
+
+# ------------------------------------------------------------ objectives ---
+@pytest.mark.parametrize("mode", [0, 1])
+def test_objective_equals_materialisation_rule(oracle_lib, mode):
+    """Lemma 1 (Eq. 4) and Eq. 6 equal the savings of the Section III-A rule."""
+    rng = np.random.default_rng(20 + mode)
+    for trial in range(40):
+        inst = wl.random_small(rng, int(rng.integers(1, 12)), int(rng.integers(1, 5)), mode)
+        prob = _prob(oracle_lib, inst)
+        pl = (rng.random((inst.W, inst.n)) < 0.4).astype(np.uint8)
+        assert oracle_lib.objective(prob, pl) == bf.materialisation_saving(inst, pl)
+
+
+def test_lemma1_reduction(oracle_lib):
+    """Setting f_{m<-h} = f_m turns Eq. 6 into Eq. 4 (end of Section III-C)."""
+    rng = np.random.default_rng(30)
+    for trial in range(40):
+        inst = wl.random_small(rng, int(rng.integers(1, 15)), int(rng.integers(1, 6)), 0)
+        src = wl.Instance(**{**inst.__dict__, "mode": 1,
+                             "transfer": np.broadcast_to(inst.transfer[None], (inst.W, inst.W, inst.n)).copy()})
+        pl = (rng.random((inst.W, inst.n)) < 0.5).astype(np.uint8)
+        assert oracle_lib.objective_F(_prob(oracle_lib, inst), pl) == \
+            oracle_lib.objective_Fpair(_prob(oracle_lib, src), pl)
+
+
+def test_theorem2_spider_closed_form(oracle_lib):
+    """Theorem 2's spider: covering the first x_i chunks of leg i saves
+    lambda_i * sum_{d<=x_i}(2d - 1) = x_i^2 / s_i; demand scaled by L = lcm(s_i)."""
+    s = [3, 4, 5, 4, 3, 5]                      # a 3-Partition instance, B = 12, q = 2
+    L = int(np.lcm.reduce(s))
+    q, B = 2, 12
+    n = sum(s)
+    parent, depth, leg = [], [], []
+    for i, si in enumerate(s):
+        for d in range(1, si + 1):
+            parent.append(-1 if d == 1 else len(parent) - 1)
+            depth.append(d)
+            leg.append(i)
+    parent = np.array(parent, np.int32)
+    depth = np.array(depth, np.int64)
+    W = q + 1                                   # q holders + one requester (the last)
+    demand = np.zeros((W, n), np.int64)
+    demand[q] = np.array([L // s[leg[b]] for b in range(n)])
+    recompute = np.tile(2 * depth, (W, 1))
+    budget = np.array([B] * q + [0], np.int32)
+    rng = np.random.default_rng(4)
+    for mode in (0, 1):
+        transfer = np.ones((W, n), np.int64) if mode == 0 else np.ones((W, W, n), np.int64)
+        inst = wl.Instance("spider", n, W, parent, np.ones(n, np.int32), demand, recompute,
+                           transfer, mode, budget, 1, 1)
+        prob = _prob(oracle_lib, inst)
+        for trial in range(20):
+            x = [int(rng.integers(0, si + 1)) for si in s]
+            pl = np.zeros((W, n), np.uint8)
+            for b in range(n):
+                if depth[b] <= x[leg[b]]:
+                    pl[int(rng.integers(q)), b] = 1       # any holder covers it
+            expect = sum(L * xi * xi // si for xi, si in zip(x, s))
+            assert oracle_lib.objective(prob, pl) == expect
+        # a valid 3-partition ({3,4,5}, {4,3,5}) reaches L * q * B
+        pl = np.zeros((W, n), np.uint8)
+        for b in range(n):
+            pl[0 if leg[b] < 3 else 1, b] = 1
+        assert oracle_lib.objective(prob, pl) == L * q * B
+
+
+# ------------------------------------------------------------- marginals ---
+@pytest.mark.parametrize("mode", [0, 1])
+def test_prop1_marginal_additivity(oracle_lib, mode):
+    """Prop. 1 / Eq. 10: G(T_-h, T') - G(T_-h, {}) = sum_{b in T'} p_h(b) for any T'."""
+    rng = np.random.default_rng(40 + mode)
+    for trial in range(40):
+        inst = wl.random_small(rng, int(rng.integers(1, 14)), int(rng.integers(1, 6)), mode)
+        prob = _prob(oracle_lib, inst)
+        pl = (rng.random((inst.W, inst.n)) < 0.4).astype(np.uint8)
+        h = int(rng.integers(inst.W))
+        p = oracle_lib.marginal(prob, h, pl)
+        pl[h] = 0
+        base = bf.materialisation_saving(inst, pl)
+        for rep in range(5):
+            Tp = (rng.random(inst.n) < 0.5).astype(np.uint8)
+            pl2 = pl.copy()
+            pl2[h] = Tp
+            assert bf.materialisation_saving(inst, pl2) - base == int(p[Tp.astype(bool)].sum())
+
+
+def test_eq10_equals_eq7_when_source_independent(oracle_lib):
+    rng = np.random.default_rng(50)
+    for trial in range(40):
+        inst = wl.random_small(rng, int(rng.integers(1, 14)), int(rng.integers(1, 6)), 0)
+        src = wl.Instance(**{**inst.__dict__, "mode": 1,
+                             "transfer": np.broadcast_to(inst.transfer[None], (inst.W, inst.W, inst.n)).copy()})
+        pl = (rng.random((inst.W, inst.n)) < 0.4).astype(np.uint8)
+        h = int(rng.integers(inst.W))
+        np.testing.assert_array_equal(oracle_lib.marginal(_prob(oracle_lib, inst), h, pl),
+                                      oracle_lib.marginal(_prob(oracle_lib, src), h, pl))
+
+
+# -------------------------------------------------- greedy / refinement ---
+@pytest.mark.parametrize("mode", [0, 1])
+def test_theorem3_half_approximation(oracle_lib, mode):
+    """Theorem 3: one fixed-order greedy pass reaches >= OPT / 2; refinement and
+    starts never go below it and never above OPT."""
+    rng = np.random.default_rng(60 + mode)
+    for trial in range(12):
+        W = int(rng.integers(2, 4))
+        inst = wl.random_small(rng, int(rng.integers(2, 7)), W, mode, k_max=3, w_max=2)
+        prob = _prob(oracle_lib, inst)
+        opt = bf.joint_optimum(inst)
+        orders = wl.random_orders(W, 3, seed=trial)
+        greedy = oracle_lib.plan(prob, 3, 0, orders=orders, threads=1)
+        full = oracle_lib.plan(prob, 3, 5, orders=orders, threads=1)
+        for s in range(3):
+            assert 2 * greedy.per_start_objective[s] >= opt
+            assert greedy.per_start_objective[s] <= full.per_start_objective[s] <= opt
+        assert full.objective == full.per_start_objective.max()
+        assert full.objective == bf.materialisation_saving(inst, full.placement)
+
+
+@pytest.mark.parametrize("cfg", [0, 1])
+def test_plan_invariants_on_configs(oracle_lib, cfg):
+    """Algorithm 1 on the tiny and RAG workloads: feasible, prefix-complete,
+    non-decreasing through refinement, best-of-starts, and coordinate-wise
+    optimal when the returned start converged."""
+    inst = wl.make(cfg)
+    prob = _prob(oracle_lib, inst)
+    S = inst.starts
+    greedy = oracle_lib.plan(prob, S, 0)
+    res = oracle_lib.plan(prob, S, inst.rounds)
+    assert res.objective == res.per_start_objective.max()
+    assert res.best_start == int(np.argmax(res.per_start_objective))
+    assert np.all(res.per_start_objective >= greedy.per_start_objective)
+    for m in range(inst.W):
+        assert bf.is_parent_closed(inst.parent, res.placement[m])
+        assert int(inst.weight[res.placement[m].astype(bool)].sum()) <= inst.budget[m]
+    assert oracle_lib.objective(prob, res.placement) == res.objective
+    b = res.best_start
+    if res.per_start_sweeps[b] < inst.rounds:
+        for h in range(inst.W):
+            best, p, _ = oracle_lib.worker_update(prob, h, res.placement)
+            assert best <= int(p[res.placement[h].astype(bool)].sum())
+
+
+def test_default_orders_shape(oracle_lib):
+    inst = wl.make(1)
+    prob = _prob(oracle_lib, inst)
+    o = oracle_lib.default_orders(prob, 6)
+    for s in range(6):
+        assert sorted(o[s]) == list(range(inst.W))
+    sc = oracle_lib.standalone(prob)
+    assert all(sc[o[0][t]] >= sc[o[0][t + 1]] for t in range(inst.W - 1))
+    np.testing.assert_array_equal(o[1], o[0][::-1])
+    assert list(oracle_lib.default_orders(prob, 1)[0]) == list(range(inst.W))
+
+
+# ------------------------------------------------- generator constants ---
+def test_generator_constants_match_paper_arithmetic():
+    """Fig. 1, Table I and RQ1 arithmetic that the cost generator is built on."""
+    assert wl.CHUNK_BYTES == 18_874_368                              # "18.9-MB"
+    assert round(wl.CHUNK_BYTES / 1e6, 1) == 18.9
+    t = int(wl.fetch_us(wl.CHUNK_BYTES, 1_500_000_000))              # "about 100.7 ms"
+    assert t == 100_663 and round(t / 1000, 1) == 100.7
+    b7 = 512 * 57_344                                                 # L4/A100-7B, "29.4-MB"
+    assert round(b7 / 1e6, 1) == 29.4
+    assert round(512 * 262_144 / 1e6, 1) == 134.2                    # A100-32B, "134.2-MB"
+    f7 = int(wl.fetch_us(b7, 3_000_000_000)) / 1000                   # ms at 3 Gb/s
+    p_cross = (f7 - 48.1) / 0.0050                                    # A100-7B fit
+    assert abs(p_cross - 6100) / 6100 < 0.02                          # "near 6.1K tokens"
+    assert 170.2 > f7                                                 # L4-7B "favors fetching"
+    # the middle generator class crosses the 1.5 Gb/s fetch near 3.8K tokens (Fig. 1, L4)
+    p_mid = (t - wl.BETA_US[1]) / wl.ALPHA_US_PER_TOKEN[1]
+    assert abs(p_mid - 3800) < 100
+    assert wl.ALPHA_US_PER_TOKEN[1] == 3 * wl.ALPHA_US_PER_TOKEN[0]
+    assert wl.ALPHA_US_PER_TOKEN[2] == 8 * wl.ALPHA_US_PER_TOKEN[0]
+
+
+def test_refinement_accepts_only_strict_improvements(oracle_lib):
+    """Section IV-C: only strictly improving replacements are accepted, so a
+    greedy result that is already coordinate-wise optimal ends after exactly
+    one sweep with no accepted update (the DP re-finds an equal-valued set)."""
+    rng = np.random.default_rng(70)
+    seen = 0
+    for trial in range(60):
+        mode = trial % 2
+        inst = wl.random_small(rng, int(rng.integers(3, 9)), int(rng.integers(2, 4)), mode,
+                               k_max=3, w_max=2)
+        prob = _prob(oracle_lib, inst)
+        orders = wl.random_orders(inst.W, 1, seed=trial)
+        g = oracle_lib.plan(prob, 1, 0, orders=orders, threads=1)
+        local_opt = True
+        for h in range(inst.W):
+            best, p, _ = oracle_lib.worker_update(prob, h, g.placement)
+            if best > int(p[g.placement[h].astype(bool)].sum()):
+                local_opt = False
+        r = oracle_lib.plan(prob, 1, 4, orders=orders, threads=1)
+        if local_opt:
+            seen += 1
+            assert r.per_start_sweeps[0] == 1 and r.per_start_accepted[0] == 0
+            np.testing.assert_array_equal(r.placement, g.placement)
+        else:
+            assert r.per_start_accepted[0] >= 1
+    assert seen >= 10
