@@ -1,0 +1,232 @@
+/*
+ * prefixplace.h -- C ABI of libprefixplace.so, the GB300 (sm_103a) planner
+ * hot path of PrefixPlace (arXiv 2608.01655).
+ *
+ * The library plans prefix-complete KV-cache targets for W workers over a
+ * prefix tree of n chunks.  Its hot path is the per-worker exact update of
+ * coordinate refinement: node marginals against the other workers' current
+ * targets (Eq. 10 requester-side, Eq. 7 source-dependent), then the exact
+ * capacity-k rooted-tree DP (Eq. 9, Theorem 1) and its traceback, batched over
+ * workers and order-diverse starts (Algorithm 1).
+ *
+ * Conventions shared by every entry point
+ *   - Node ids are the caller's (0..n-1).  The preorder used internally
+ *     (roots, then children, each in ascending node id) is never exposed
+ *     except through pp_instance_preorder().
+ *   - Integers only: costs are int64 microseconds, demand int64 counts.  The
+ *     paper's floating-point tolerance epsilon is therefore 0: a refinement
+ *     update is accepted only on a strict improvement.
+ *   - Every function returns a pp_status and never aborts; pp_last_error()
+ *     gives a thread-local message for the last failure in the calling
+ *     thread.  Kernels report device-side problems (a budget above the
+ *     declared bound, a wait that ran out) through a status word of the
+ *     instance; pp_instance_sync() and pp_plan_run() read and clear it.
+ *   - "device" pointers are CUDA global-memory pointers of the instance's
+ *     device (for example torch tensors' data_ptr()); "host" pointers are
+ *     ordinary CPU memory.  The caller owns every buffer it passes; the
+ *     library owns the instance and its internal scratch.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls that
+ *     take device buffers are asynchronous and stream-ordered.
+ *   - Limits: 1 <= W <= 32 workers (holder sets are 32-bit masks), the
+ *     largest useful budget min(k, total chunk weight) <= 32768 slots, and a
+ *     skip-row stack depth (bounded by the tree depth) <= 65533.
+ */
+#ifndef PREFIXPLACE_H
+#define PREFIXPLACE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pp_instance pp_instance;   /* opaque, library-owned */
+
+typedef enum {
+    PP_OK = 0,
+    PP_EINVAL = 1,      /* bad argument: size, mode, null pointer, weight < 1, negative data */
+    PP_ENOTTREE = 2,    /* parent[] out of range, self-parent, or a cycle */
+    PP_EOVERFLOW = 3,   /* sum_b sum_m demand * recompute exceeds 2^62 */
+    PP_ENOMEM = 4,      /* device or host allocation failed */
+    PP_ECUDA = 5,       /* a CUDA runtime call failed */
+    PP_ETIMEOUT = 6,    /* a bounded device-side wait ran out (device status word) */
+    PP_EBOUNDS = 7      /* a device-side bounds check failed (device status word) */
+} pp_status;
+
+enum { PP_TRANSFER_REQUESTER = 0, PP_TRANSFER_SOURCE = 1 };
+
+/* Optional outputs of pp_plan_run.  Array members may be NULL. */
+typedef struct {
+    int64_t *per_start_objective;  /* [n_starts] host, out: objective of each candidate */
+    int32_t *per_start_sweeps;     /* [n_starts] host, out: refinement sweeps run */
+    int32_t *per_start_accepted;   /* [n_starts] host, out: accepted refinement updates */
+    int32_t *orders_used;          /* [n_starts][W] host, out: the start orders */
+    int32_t best_start;            /* out: index of the returned candidate */
+    int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded) */
+    int64_t dp_cells;              /* out: sum over executed DPs of n * k_h (Eq. 9 cells) */
+    int32_t kernel_launches;       /* out: kernels launched by this call */
+} pp_plan_stats;
+
+/*
+ * pp_instance_create -- validate a planner instance, upload it and build the
+ * per-instance tables (preorder, next(i), the DP's row metadata, and the
+ * gains of Eq. 2-3 or Eq. 5).
+ *
+ *   n, W          chunks (n >= 0) and workers (1..32)
+ *   parent        host [n]: parent node id, or -1 for a child of the implicit
+ *                 no-cost dummy root (Section III-A)
+ *   weight        host [n]: budget slots per chunk, >= 1 (1 = the paper's
+ *                 equal-sized chunks)
+ *   demand        host [W][n]: Lambda_m(b) >= 0, already counted on every
+ *                 chunk of each request's prefix path (Section III-A)
+ *   recompute     host [W][n]: w_m(b) >= 0 in microseconds
+ *   transfer      host, >= 0 microseconds: mode PP_TRANSFER_REQUESTER
+ *                 [W][n] f_m(b) (Eq. 1); mode PP_TRANSFER_SOURCE [W][W][n],
+ *                 element [h][m][b] = f_{m<-h}(b) (Section III-C); the
+ *                 diagonal h == m is never read
+ *   budget        host [W]: k_m >= 0 slots
+ *   stream        stream for the uploads and precompute kernels
+ *   out           receives the instance (NULL on failure)
+ * Errors: PP_EINVAL, PP_ENOTTREE, PP_EOVERFLOW (sum_b sum_m Lambda * w,
+ * computed exactly, above 2^62; this bound keeps every objective, marginal
+ * and DP value of the instance inside int64), PP_ENOMEM, PP_ECUDA.
+ * The call synchronises `stream` before returning; the inputs are not retained.
+ */
+pp_status pp_instance_create(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
+                             const int64_t *demand, const int64_t *recompute,
+                             const int64_t *transfer, int32_t transfer_mode,
+                             const int32_t *budget, void *stream, pp_instance **out);
+
+/* Frees the instance and its device memory.  NULL is accepted. */
+pp_status pp_instance_destroy(pp_instance *inst);
+
+/*
+ * pp_instance_preorder -- the internal preorder (Section IV-A, "number nodes
+ * in preorder and compute next(i)"): order[i] = node at 0-based position i,
+ * next[i] = first position after that node's subtree.  Host [n] outputs.
+ * Also reports the depth of the DP's skip-row stack (may be NULL).
+ */
+pp_status pp_instance_preorder(const pp_instance *inst, int32_t *order, int32_t *next,
+                               int32_t *stack_depth);
+
+/*
+ * pp_row_plan -- host-only (no CUDA call): the preorder and the DP's row plan
+ * for a parent array, as pp_instance_create builds them.  Positions are swept
+ * from n-1 down to 0; the skip branch of Eq. 9 at position i reads row
+ * next(i), which is the row just computed when next(i) == i + 1 (skip_code
+ * -1), the zero boundary row when next(i) == n (skip_code -2), and otherwise
+ * a row saved on the skip-row stack at level skip_code >= 0.  push_level[i]
+ * >= 0 saves row i at that level; -1 saves nothing.
+ *   order, next, skip_code, push_level   host [n] out
+ *   stack_depth                          host out: levels used
+ * Errors: PP_EINVAL, PP_ENOTTREE.
+ */
+pp_status pp_row_plan(int32_t n, const int32_t *parent, int32_t *order, int32_t *next,
+                      int32_t *skip_code, int32_t *push_level, int32_t *stack_depth);
+
+/*
+ * pp_instance_sync -- synchronise `stream`, then read and clear the device
+ * status word.  Returns PP_OK, PP_ETIMEOUT, PP_EBOUNDS or PP_ECUDA.
+ */
+pp_status pp_instance_sync(pp_instance *inst, void *stream);
+
+/*
+ * pp_marginals -- exact node marginals of one worker per batch item against
+ * the other workers' targets (Prop. 1).
+ *   requester-side: p_h(b) = a_h(b) + 1{no worker l != h holds b} Delta(b)   (Eq. 10)
+ *   source-dependent: p_h(b) = sum_m Lambda_m(b) [q_{m<-h}(b) - v_m^{(-h)}(b)]_+ (Eq. 7)
+ *     with v_m^{(-h)}(b) the best q_{m<-l}(b) over holders l != h (0 if none).
+ *   batch         items (>= 0)
+ *   worker        device [batch]: h per item, 0..W-1
+ *   holder_mask   device [batch][n] by node id: bit l set = worker l holds the
+ *                 chunk; bit h itself is ignored
+ *   profit        device [batch][n] by node id, out
+ * Errors: PP_EINVAL (host-side argument checks).  A worker id out of range
+ * sets PP_EBOUNDS in the status word and leaves that item's profits at 0.
+ */
+pp_status pp_marginals(pp_instance *inst, int32_t batch, const int32_t *worker,
+                       const uint32_t *holder_mask, int64_t *profit, void *stream);
+
+/*
+ * pp_dp_bits_size -- bytes of the decision-bit workspace that pp_tree_dp
+ * writes and pp_traceback reads for `batch` items whose budgets are at most
+ * `max_budget`.  Returns 0 for batch <= 0 or an invalid max_budget.
+ */
+size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_t max_budget);
+
+/*
+ * pp_tree_dp -- the exact capacity-k prefix-complete tree knapsack (Eq. 9,
+ * Theorem 1) for each batch item:
+ *   D[i][0] = 0, D[n][j] = 0,
+ *   D[i][j] = max{ D[next(i)][j], p(b_i) + D[i+1][j - w_i] }  (take needs j >= w_i)
+ * over preorder positions i, recording "take" only on a strict improvement.
+ *   profit        device [batch][n] by node id; any int64 values whose
+ *                 absolute sum stays below 2^62 (not checked)
+ *   budget        device [batch]: k per item, 0 <= k <= max_budget
+ *   max_budget    host: upper bound of budget[]; fixes the bit layout
+ *   best          device [batch], out: D[0][k]
+ *   bits          device workspace of pp_dp_bits_size(inst, batch, max_budget)
+ *                 bytes, out: decision bits for pp_traceback
+ * A budget outside [0, max_budget] sets PP_EBOUNDS and that item's best to 0.
+ * The call may allocate instance-owned device scratch for the skip-row stack
+ * on first use (or when a larger batch needs more).
+ */
+pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t *profit,
+                     const int32_t *budget, int32_t max_budget, int64_t *best,
+                     uint32_t *bits, void *stream);
+
+/*
+ * pp_traceback -- recover each item's optimal parent-closed set from the
+ * decision bits (Algorithm 1, "backtrack from D[1,k]"): start at position 0
+ * with j = k; "take" marks the chunk, j -= w_i and moves to i+1; "skip" moves
+ * to next(i).  Among optimal sets this returns the lexicographically smallest
+ * preorder indicator.
+ *   bits, budget, max_budget   exactly as given to pp_tree_dp
+ *   chosen        device [batch][n] by node id, out: 1 = selected, else 0
+ */
+pp_status pp_traceback(pp_instance *inst, int32_t batch, const uint32_t *bits,
+                       const int32_t *budget, int32_t max_budget, uint8_t *chosen,
+                       void *stream);
+
+/*
+ * pp_objective -- the planner objective of each batch item's placement:
+ * F (Lemma 1, Eq. 4) for requester-side instances, F_pair (Eq. 6) for
+ * source-dependent ones.  Placements need not be feasible.
+ *   chosen        device [batch][W][n] by node id: nonzero = worker holds chunk
+ *   obj           device [batch], out
+ */
+pp_status pp_objective(pp_instance *inst, int32_t batch, const uint8_t *chosen, int64_t *obj,
+                       void *stream);
+
+/*
+ * pp_plan_run -- Algorithm 1 (procedure PrefixPlace) without the
+ * requester-side safeguard candidates: for each start order, one
+ * WorkerGreedy pass (Theorem 3), then at most max_rounds refinement sweeps;
+ * a sweep with no accepted update ends that start.  Starts run batched.
+ *   n_starts      S >= 1
+ *   orders        host [S][W] permutations of 0..W-1, or NULL for the default:
+ *                 S == 1 the identity; otherwise start 0 = standalone-score
+ *                 order (descending, ties to the lower id), start 1 its
+ *                 reverse, start s >= 2 a Fisher-Yates shuffle driven by
+ *                 SplitMix64 seeded with s (j = next() mod (i + 1), i = W-1..1)
+ *   max_rounds    R >= 0 refinement sweeps
+ *   placement     host [W][n] out: the best candidate (highest objective,
+ *                 ties to the lowest start), 1 = resident
+ *   objective     host out: its objective (Eq. 4 or Eq. 6)
+ *   stats         optional (NULL) extra outputs
+ * Synchronous: returns after the result is on the host.  Errors: PP_EINVAL,
+ * PP_ENOMEM, PP_ECUDA, and any device status (PP_ETIMEOUT, PP_EBOUNDS).
+ */
+pp_status pp_plan_run(pp_instance *inst, int32_t n_starts, const int32_t *orders,
+                      int32_t max_rounds, uint8_t *placement, int64_t *objective,
+                      pp_plan_stats *stats, void *stream);
+
+/* Thread-local description of the last failure in this thread ("" if none). */
+const char *pp_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PREFIXPLACE_H */

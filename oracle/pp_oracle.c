@@ -18,8 +18,9 @@
  *   f_m(b)       fetch cost, requester-side                   (Eq. 1)
  *   f_{m<-h}(b)  fetch cost from holder h, source-dependent   (Section III-C)
  *   k_m          budget of worker m in slots
- * Chunks may occupy more than one slot ("weight"); the paper's unit-size
- * chunks are the special case weight == 1 (reading stated in the design doc).
+ * Chunks may occupy more than one slot ("weight"); the take branch of Eq. 9
+ * then spends w_i slots and needs j >= w_i.  The paper's equal-sized chunks
+ * are the special case weight == 1.
  *
  * Functions and the passage each one follows:
  *   or_preorder        Section IV-A: preorder b_1..b_n and next(i)
@@ -487,6 +488,8 @@ int32_t or_plan(const or_inst *I, int32_t S, const int32_t *orders, int32_t R, i
         if (per_start_accepted) per_start_accepted[s] = st[s].accepted;
         cells += st[s].cells;
     }
+    if (!orders && S > 1)                      /* the standalone-score DPs of the default orders */
+        for (int32_t m = 0; m < W; ++m) cells += (int64_t)n * I->budget[m];
     if (cells_out) *cells_out = cells;
     memcpy(placement, st[best].T, (size_t)W * n);
     *objective = st[best].objective;

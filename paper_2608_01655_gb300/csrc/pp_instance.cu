@@ -1,0 +1,385 @@
+// Instance set-up: validation, preorder (Section IV-A), the DP's skip-row
+// stack plan, and the gain tables of Eq. 2-3 (requester-side) or Eq. 5
+// (source-dependent) computed on the device.
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "pp_internal.cuh"
+
+namespace pp {
+
+static thread_local std::string g_last_error;
+
+pp_status fail(pp_status s, const std::string &msg)
+{
+    g_last_error = msg;
+    return s;
+}
+
+pp_status cuda_fail(cudaError_t e, const char *what)
+{
+    g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+    return e == cudaErrorMemoryAllocation ? PP_ENOMEM : PP_ECUDA;
+}
+
+pp_status ensure_scratch(Scratch &s, size_t bytes)
+{
+    if (s.bytes >= bytes && s.ptr) return PP_OK;
+    free_scratch(s);
+    if (bytes == 0) return PP_OK;
+    cudaError_t e = cudaMalloc(&s.ptr, bytes);
+    if (e != cudaSuccess) {
+        s.ptr = nullptr;
+        return cuda_fail(e, "cudaMalloc(scratch)");
+    }
+    s.bytes = bytes;
+    return PP_OK;
+}
+
+void free_scratch(Scratch &s)
+{
+    if (s.ptr) cudaFree(s.ptr);
+    s.ptr = nullptr;
+    s.bytes = 0;
+}
+
+bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g)
+{
+    if (max_budget < 0) return false;
+    int64_t k = max_budget;
+    if (k > inst->total_weight) k = inst->total_weight;   // larger budgets change nothing
+    int C = 1;
+    while ((int64_t)C * 1024 < k) C *= 2;
+    if (C > 32) return false;
+    int T = (int)((k + C - 1) / C);
+    T = (T + 31) / 32 * 32;
+    if (T < 32) T = 32;
+    g->C = C;
+    g->T = T;
+    g->kpad = T * C;
+    g->words = g->kpad / 32;
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// Preorder with roots first and children in ascending node id; next(i) is the
+// first position after the subtree at position i.  Returns false if parent[]
+// is not a forest.
+// ---------------------------------------------------------------------------
+static bool build_preorder(int32_t n, const int32_t *parent, std::vector<int32_t> &order,
+                           std::vector<int32_t> &next)
+{
+    std::vector<int32_t> head(n + 1, -1), sib(n, -1), stack;
+    // children lists in ascending id: insert in descending id at the head
+    for (int32_t v = n - 1; v >= 0; --v) {
+        int32_t p = parent[v] < 0 ? n : parent[v];
+        sib[v] = head[p];
+        head[p] = v;
+    }
+    order.assign(n, 0);
+    next.assign(n, 0);
+    std::vector<int32_t> pos(n, -1);
+    int32_t cnt = 0;
+    // iterative DFS: a stack of "next child to visit" cursors
+    std::vector<int32_t> cursor;
+    cursor.push_back(head[n]);
+    std::vector<int32_t> path;     // nodes whose subtree is open
+    while (!cursor.empty()) {
+        int32_t c = cursor.back();
+        if (c < 0) {
+            cursor.pop_back();
+            if (!path.empty()) {
+                int32_t u = path.back();
+                path.pop_back();
+                next[pos[u]] = cnt;
+            }
+            continue;
+        }
+        cursor.back() = sib[c];
+        pos[c] = cnt;
+        order[cnt++] = c;
+        path.push_back(c);
+        cursor.push_back(head[c]);
+        if ((int32_t)path.size() > n) return false;
+    }
+    return cnt == n;
+}
+
+// Skip-row stack plan: see the DP row metadata comment in pp_internal.cuh.
+static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vector<int32_t> &meta,
+                           int32_t *depth_out)
+{
+    meta.assign(n, 0);
+    // last_reader[r] = smallest q with next(q) == r and q < r - 1 (stack reads only)
+    std::vector<int32_t> last_reader(n + 1, -1);
+    for (int32_t q = n - 1; q >= 0; --q) {
+        int32_t r = next[q];
+        if (r != q + 1 && r != n) last_reader[r] = q;
+    }
+    std::vector<int32_t> level(n + 1, -1);
+    int32_t depth = 0, maxd = 0;
+    for (int32_t i = n - 1; i >= 0; --i) {
+        int32_t r = next[i];
+        int skip;
+        if (r == i + 1) skip = kSkipCur;
+        else if (r == n) skip = kSkipZero;
+        else {
+            skip = level[r];
+            if (skip < 0) return false;
+            if (last_reader[r] == i) {          // last reader: pop
+                --depth;
+                if (level[r] != depth) return false;
+            }
+        }
+        int push = -1;
+        if (i >= 1 && last_reader[i] >= 0) {
+            push = depth;
+            level[i] = depth++;
+            if (depth > maxd) maxd = depth;
+            if (depth > kMaxStackLevels) return false;
+        }
+        meta[i] = meta_pack(skip, push);
+    }
+    *depth_out = maxd;
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// Gain tables (one-time precompute, preorder-indexed):
+//   mode 0: a[m][i] = Lambda_m(b) min{w_m(b), f_m(b)}            (Eq. 2)
+//           Delta[i] = sum_m Lambda_m(b) [w_m(b) - f_m(b)]_+       (Eq. 3)
+//   mode 1: g[h][m][i] = Lambda_m(b) q_{m<-h}(b)                   (Eq. 5)
+// with b = order[i].  Lambda >= 0 commutes with min, max and [.]_+, so Eq. 7
+// can be evaluated on these products exactly.
+// ---------------------------------------------------------------------------
+__global__ void k_gain_requester(int32_t n, int32_t W, const int32_t *__restrict__ order,
+                                 const int64_t *__restrict__ demand,
+                                 const int64_t *__restrict__ recompute,
+                                 const int64_t *__restrict__ transfer, int64_t *__restrict__ a,
+                                 int64_t *__restrict__ delta)
+{
+    for (int32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        int32_t b = order[i];
+        int64_t d = 0;
+        for (int32_t m = 0; m < W; ++m) {
+            size_t o = (size_t)m * n + b;
+            int64_t lam = demand[o], w = recompute[o], f = transfer[o];
+            a[(size_t)m * n + i] = lam * (w < f ? w : f);
+            d += lam * (w > f ? w - f : 0);
+        }
+        delta[i] = d;
+    }
+}
+
+__global__ void k_gain_source(int32_t n, int32_t W, const int32_t *__restrict__ order,
+                              const int64_t *__restrict__ demand,
+                              const int64_t *__restrict__ recompute,
+                              const int64_t *__restrict__ transfer, int64_t *__restrict__ g)
+{
+    const int32_t hm = blockIdx.y;               // h * W + m
+    const int32_t h = hm / W, m = hm % W;
+    for (int32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        int32_t b = order[i];
+        int64_t lam = demand[(size_t)m * n + b], w = recompute[(size_t)m * n + b];
+        int64_t q;
+        if (h == m) q = w;
+        else {
+            int64_t f = transfer[(size_t)hm * n + b];
+            q = w > f ? w - f : 0;
+        }
+        g[(size_t)hm * n + i] = lam * q;
+    }
+}
+
+}  // namespace pp
+
+using namespace pp;
+
+extern "C" const char *pp_last_error(void) { return g_last_error.c_str(); }
+
+extern "C" pp_status pp_instance_destroy(pp_instance *inst)
+{
+    if (!inst) return PP_OK;
+    int cur = 0;
+    cudaGetDevice(&cur);
+    cudaSetDevice(inst->device);
+    cudaFree(inst->d_order);
+    cudaFree(inst->d_next);
+    cudaFree(inst->d_wpre);
+    cudaFree(inst->d_meta);
+    cudaFree(inst->d_budget);
+    cudaFree(inst->d_a);
+    cudaFree(inst->d_delta);
+    cudaFree(inst->d_g);
+    cudaFree(inst->d_status);
+    free_scratch(inst->stack);
+    free_scratch(inst->plan);
+    free_scratch(inst->plan_bits);
+    cudaSetDevice(cur);
+    delete inst;
+    return PP_OK;
+}
+
+template <typename T>
+static pp_status upload(T **dst, const T *src, size_t count, cudaStream_t st)
+{
+    PP_CUDA(cudaMalloc((void **)dst, sizeof(T) * (count ? count : 1)));
+    if (count) PP_CUDA(cudaMemcpyAsync(*dst, src, sizeof(T) * count, cudaMemcpyHostToDevice, st));
+    return PP_OK;
+}
+
+static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
+                             const int64_t *demand, const int64_t *recompute,
+                             const int64_t *transfer, int32_t mode, const int32_t *budget,
+                             cudaStream_t st, pp_instance *inst)
+{
+    if (n < 0) return fail(PP_EINVAL, "n must be >= 0");
+    if (W < 1 || W > 32) return fail(PP_EINVAL, "W must be in 1..32");
+    if (mode != PP_TRANSFER_REQUESTER && mode != PP_TRANSFER_SOURCE)
+        return fail(PP_EINVAL, "transfer_mode must be 0 (requester) or 1 (source)");
+    if (!budget || (n > 0 && (!parent || !weight || !demand || !recompute || !transfer)))
+        return fail(PP_EINVAL, "null input pointer");
+    for (int32_t m = 0; m < W; ++m)
+        if (budget[m] < 0) return fail(PP_EINVAL, "budget must be >= 0");
+    for (int32_t v = 0; v < n; ++v) {
+        if (parent[v] < -1 || parent[v] >= n || parent[v] == v)
+            return fail(PP_ENOTTREE, "parent id out of range or self-parent at node " + std::to_string(v));
+        if (weight[v] < 1) return fail(PP_EINVAL, "chunk weight must be >= 1");
+    }
+    const size_t Wn = (size_t)W * n;
+    const size_t tn = mode == PP_TRANSFER_SOURCE ? (size_t)W * Wn : Wn;
+    __int128 total = 0;
+    for (size_t x = 0; x < Wn; ++x) {
+        if (demand[x] < 0 || recompute[x] < 0) return fail(PP_EINVAL, "negative demand or recompute cost");
+        total += (__int128)demand[x] * (__int128)recompute[x];
+    }
+    for (size_t x = 0; x < tn; ++x)
+        if (transfer[x] < 0) return fail(PP_EINVAL, "negative transfer cost");
+    if (total > ((__int128)1 << 62))
+        return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
+
+    inst->n = n;
+    inst->W = W;
+    inst->mode = mode;
+    if (!build_preorder(n, parent, inst->h_order, inst->h_next))
+        return fail(PP_ENOTTREE, "parent array contains a cycle");
+    if (!build_row_meta(n, inst->h_next, inst->h_meta, &inst->stack_depth))
+        return fail(PP_EINVAL, "skip-row stack deeper than supported");
+    inst->h_wpre.resize(n);
+    inst->total_weight = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        inst->h_wpre[i] = weight[inst->h_order[i]];
+        inst->total_weight += weight[i];
+    }
+    inst->h_budget.assign(budget, budget + W);
+
+    PP_CUDA(cudaGetDevice(&inst->device));
+    PP_CUDA(cudaDeviceGetAttribute(&inst->sm_count, cudaDevAttrMultiProcessorCount, inst->device));
+    pp_status s;
+    if ((s = upload(&inst->d_order, inst->h_order.data(), n, st))) return s;
+    if ((s = upload(&inst->d_next, inst->h_next.data(), n, st))) return s;
+    if ((s = upload(&inst->d_wpre, inst->h_wpre.data(), n, st))) return s;
+    if ((s = upload(&inst->d_meta, inst->h_meta.data(), n, st))) return s;
+    if ((s = upload(&inst->d_budget, budget, W, st))) return s;
+    PP_CUDA(cudaMalloc(&inst->d_status, sizeof(int32_t)));
+    PP_CUDA(cudaMemsetAsync(inst->d_status, 0, sizeof(int32_t), st));
+
+    int64_t *d_dem = nullptr, *d_rec = nullptr, *d_tr = nullptr;
+    if ((s = upload(&d_dem, demand, Wn, st))) return s;
+    if ((s = upload(&d_rec, recompute, Wn, st))) { cudaFree(d_dem); return s; }
+    if ((s = upload(&d_tr, transfer, tn, st))) { cudaFree(d_dem); cudaFree(d_rec); return s; }
+    cudaError_t e = cudaSuccess;
+    int blocks = (int)((n + 255) / 256);
+    if (blocks > 4 * inst->sm_count) blocks = 4 * inst->sm_count;
+    if (blocks < 1) blocks = 1;
+    if (mode == PP_TRANSFER_REQUESTER) {
+        e = cudaMalloc(&inst->d_a, sizeof(int64_t) * (Wn ? Wn : 1));
+        if (e == cudaSuccess) e = cudaMalloc(&inst->d_delta, sizeof(int64_t) * (n ? n : 1));
+        if (e == cudaSuccess && n > 0)
+            k_gain_requester<<<blocks, 256, 0, st>>>(n, W, inst->d_order, d_dem, d_rec, d_tr,
+                                                     inst->d_a, inst->d_delta);
+    } else {
+        e = cudaMalloc(&inst->d_g, sizeof(int64_t) * (tn ? tn : 1));
+        if (e == cudaSuccess && n > 0) {
+            dim3 grid((unsigned)((blocks + W * W - 1) / (W * W) + 1), (unsigned)(W * W));
+            k_gain_source<<<grid, 256, 0, st>>>(n, W, inst->d_order, d_dem, d_rec, d_tr, inst->d_g);
+        }
+    }
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    cudaFree(d_dem);
+    cudaFree(d_rec);
+    cudaFree(d_tr);
+    if (e != cudaSuccess) return cuda_fail(e, "gain precompute");
+    return PP_OK;
+}
+
+extern "C" pp_status pp_instance_create(int32_t n, int32_t W, const int32_t *parent,
+                                        const int32_t *weight, const int64_t *demand,
+                                        const int64_t *recompute, const int64_t *transfer,
+                                        int32_t transfer_mode, const int32_t *budget, void *stream,
+                                        pp_instance **out)
+{
+    if (!out) return fail(PP_EINVAL, "out is null");
+    *out = nullptr;
+    pp_instance *inst = new (std::nothrow) pp_instance();
+    if (!inst) return fail(PP_ENOMEM, "host allocation failed");
+    pp_status s = create_impl(n, W, parent, weight, demand, recompute, transfer, transfer_mode,
+                              budget, (cudaStream_t)stream, inst);
+    if (s != PP_OK) {
+        pp_instance_destroy(inst);
+        return s;
+    }
+    *out = inst;
+    return PP_OK;
+}
+
+extern "C" pp_status pp_instance_preorder(const pp_instance *inst, int32_t *order, int32_t *next,
+                                          int32_t *stack_depth)
+{
+    if (!inst) return fail(PP_EINVAL, "null instance");
+    if (inst->n > 0 && (!order || !next)) return fail(PP_EINVAL, "null output");
+    if (inst->n > 0) {
+        std::memcpy(order, inst->h_order.data(), sizeof(int32_t) * inst->n);
+        std::memcpy(next, inst->h_next.data(), sizeof(int32_t) * inst->n);
+    }
+    if (stack_depth) *stack_depth = inst->stack_depth;
+    return PP_OK;
+}
+
+extern "C" pp_status pp_row_plan(int32_t n, const int32_t *parent, int32_t *order, int32_t *next,
+                                 int32_t *skip_code, int32_t *push_level, int32_t *stack_depth)
+{
+    if (n < 0) return fail(PP_EINVAL, "n must be >= 0");
+    if (n > 0 && (!parent || !order || !next || !skip_code || !push_level))
+        return fail(PP_EINVAL, "null pointer");
+    for (int32_t v = 0; v < n; ++v)
+        if (parent[v] < -1 || parent[v] >= n || parent[v] == v)
+            return fail(PP_ENOTTREE, "parent id out of range or self-parent at node " + std::to_string(v));
+    std::vector<int32_t> o, nx, meta;
+    if (!build_preorder(n, parent, o, nx)) return fail(PP_ENOTTREE, "parent array contains a cycle");
+    int32_t depth = 0;
+    if (!build_row_meta(n, nx, meta, &depth)) return fail(PP_EINVAL, "skip-row stack deeper than supported");
+    for (int32_t i = 0; i < n; ++i) {
+        order[i] = o[i];
+        next[i] = nx[i];
+        skip_code[i] = meta_skip(meta[i]);
+        push_level[i] = meta_push(meta[i]);
+    }
+    if (stack_depth) *stack_depth = depth;
+    return PP_OK;
+}
+
+extern "C" pp_status pp_instance_sync(pp_instance *inst, void *stream)
+{
+    if (!inst) return fail(PP_EINVAL, "null instance");
+    PP_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+    int32_t v = 0;
+    PP_CUDA(cudaMemcpy(&v, inst->d_status, sizeof(v), cudaMemcpyDeviceToHost));
+    PP_CUDA(cudaMemset(inst->d_status, 0, sizeof(int32_t)));
+    if (v == PP_ETIMEOUT) return fail(PP_ETIMEOUT, "a bounded device wait ran out");
+    if (v == PP_EBOUNDS) return fail(PP_EBOUNDS, "device bounds check failed (budget or worker id)");
+    if (v != 0) return fail(PP_ECUDA, "unknown device status " + std::to_string(v));
+    return PP_OK;
+}

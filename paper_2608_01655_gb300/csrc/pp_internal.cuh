@@ -1,0 +1,132 @@
+// Internal declarations of libprefixplace (not installed, not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "prefixplace.h"
+
+namespace pp {
+
+// ---------------------------------------------------------------------------
+// DP row metadata.  Rows are preorder positions, swept from n-1 down to 0.
+// The skip branch of Eq. 9 reads row next(i):
+//   kSkipCur   next(i) == i + 1: the row just computed (kept in registers)
+//   kSkipZero  next(i) == n: the boundary row D[n][.] = 0
+//   level >= 0 a row saved earlier on the skip-row stack at that level
+// A row is pushed only when a position q < r - 1 reads it (next(q) == r),
+// so the stack holds one row per pending subtree continuation and its depth
+// is bounded by the tree depth.
+// Packed in one int32: low 16 bits skip code + 2, high 16 bits push level + 1.
+// ---------------------------------------------------------------------------
+constexpr int kSkipZero = -2;
+constexpr int kSkipCur = -1;
+constexpr int kMaxStackLevels = 65533;
+
+__host__ __device__ inline int meta_skip(int32_t m) { return (m & 0xFFFF) - 2; }
+__host__ __device__ inline int meta_push(int32_t m) { return ((m >> 16) & 0xFFFF) - 1; }
+inline int32_t meta_pack(int skip, int push)
+{
+    return (int32_t)(((uint32_t)(push + 1) << 16) | (uint32_t)(skip + 2));
+}
+
+// Column geometry of one DP launch: thread t of the chain owns columns
+// t*C + c + 1 (c = 0..C-1); column 0 is the boundary D[.][0] = 0.  Decision
+// bits of row i are kpad/32 words; word (t/32)*C + c holds bit (t%32) for the
+// column t*C + c + 1, i.e. one __ballot_sync per (warp, c).
+struct DpGeom {
+    int C = 1;        // columns per thread
+    int T = 32;       // threads per chain
+    int kpad = 32;    // T * C columns
+    int words = 1;    // decision words per row (kpad / 32)
+};
+
+// Status word values written by kernels (same numbering as pp_status).
+constexpr int32_t kDevOk = PP_OK;
+
+struct Scratch {
+    void *ptr = nullptr;
+    size_t bytes = 0;
+};
+
+}  // namespace pp
+
+struct pp_instance {
+    int32_t n = 0;
+    int32_t W = 0;
+    int32_t mode = 0;
+    int device = 0;
+    int sm_count = 0;
+    int32_t stack_depth = 0;            // skip-row stack levels needed by the DP
+    int64_t total_weight = 0;           // sum of chunk weights
+    std::vector<int32_t> h_order, h_next, h_budget, h_wpre, h_meta;
+    // device tables, preorder-indexed unless noted
+    int32_t *d_order = nullptr;         // [n] position -> node id
+    int32_t *d_next = nullptr;          // [n]
+    int32_t *d_wpre = nullptr;          // [n] chunk weight
+    int32_t *d_meta = nullptr;          // [n] packed skip / push codes
+    int32_t *d_budget = nullptr;        // [W]
+    int64_t *d_a = nullptr;             // mode 0: [W][n] a_m(b)       (Eq. 2)
+    int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)
+    int64_t *d_g = nullptr;             // mode 1: [W][W][n] Lambda_m(b) q_{m<-h}(b) at [h][m][i] (Eq. 5)
+    int32_t *d_status = nullptr;        // device status word
+    pp::Scratch stack;                  // skip-row stack spill of pp_tree_dp
+    pp::Scratch plan;                   // pp_plan_run working set
+    pp::Scratch plan_bits;              // pp_plan_run decision bits
+};
+
+namespace pp {
+
+// error reporting (thread-local message)
+pp_status fail(pp_status s, const std::string &msg);
+pp_status cuda_fail(cudaError_t e, const char *what);
+#define PP_CUDA(call)                                                   \
+    do {                                                                \
+        cudaError_t e_ = (call);                                        \
+        if (e_ != cudaSuccess) return ::pp::cuda_fail(e_, #call);       \
+    } while (0)
+
+pp_status ensure_scratch(Scratch &s, size_t bytes);
+void free_scratch(Scratch &s);
+
+// DP launch geometry for a given largest budget (after clamping to the
+// instance's total weight).  Returns false when the budget is too large.
+bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g);
+
+// Launchers used by both the ABI calls and the planner.
+//   prof_by_node: profits indexed by node id (ABI) instead of preorder
+//   item_budget:  [batch] budgets; item_active: [batch] or null (0 = skip item)
+pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool prof_by_node,
+                         const int32_t *item_budget, const int32_t *item_active,
+                         const DpGeom &g, int64_t *best, uint32_t *bits, cudaStream_t st,
+                         int32_t max_budget);
+
+pp_status launch_marginals(pp_instance *inst, int batch, const int32_t *worker,
+                           const uint32_t *mask, bool by_node, const int32_t *item_active,
+                           int64_t *profit, int64_t *oldsum, cudaStream_t st);
+
+pp_status launch_objective(pp_instance *inst, int batch, const uint32_t *mask,
+                           const uint8_t *chosen, int64_t *obj, cudaStream_t st);
+
+// Traceback of pp_tree_dp's bits.  With mask == nullptr it writes chosen[]
+// bytes by node id (ABI); otherwise it is the planner's accept-and-update
+// step (see pp_plan.cu) and writes holder-mask bits in preorder.
+struct AcceptArgs {
+    const int32_t *worker = nullptr;    // [batch] h per item
+    const int64_t *best = nullptr;      // [batch] D[0][k]
+    const int64_t *oldsum = nullptr;    // [batch] sum of p_h over the current T_h
+    int32_t *active = nullptr;          // [batch] start still refining
+    int32_t *improved = nullptr;        // [batch] set on an accepted update
+    int32_t *accepted = nullptr;        // [batch] accepted-update counter
+    uint32_t *mask = nullptr;           // [batch][n] holder masks (preorder)
+    int greedy = 0;                     // 1: always accept (WorkerGreedy pass)
+};
+pp_status launch_traceback(pp_instance *inst, int batch, const uint32_t *bits, const DpGeom &g,
+                           const int32_t *item_budget, uint8_t *chosen, const AcceptArgs *acc,
+                           cudaStream_t st);
+
+}  // namespace pp

@@ -1,0 +1,269 @@
+// pp_plan_run: Algorithm 1 (procedure PrefixPlace) with the S start orders as
+// the batch axis.  Each step t processes worker pi_s[t] of every start s at
+// once:  marginals (Eq. 10 / Eq. 7) -> tree DP (Eq. 9) -> traceback with the
+// accept-and-update test fused in.  The greedy pass always accepts
+// (WorkerGreedy, Theorem 3); a refinement sweep accepts only strict
+// improvements (Section IV-C), and a start whose sweep accepted nothing stops
+// (its later kernels return at once).  Holder sets live on the device as one
+// 32-bit mask per chunk and start, in preorder.
+#include <algorithm>
+#include <cstring>
+#include <numeric>
+
+#include "pp_internal.cuh"
+
+namespace pp {
+
+// per-sweep bookkeeping: a start that accepted nothing is done
+__global__ void k_sweep_end(int S, int32_t *active, const int32_t *improved, int32_t *sweeps)
+{
+    int s = blockIdx.x * blockDim.x + threadIdx.x;
+    if (s < S && active[s]) {
+        sweeps[s] += 1;
+        active[s] = improved[s];
+    }
+}
+
+// SplitMix64 (Steele, Lea and Flood, OOPSLA 2014)
+static uint64_t splitmix64(uint64_t &x)
+{
+    uint64_t z = (x += 0x9E3779B97F4A7C15ULL);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+struct PlanBuffers {
+    uint32_t *mask;      // [B][n]
+    int64_t *profit;     // [B][n]
+    int64_t *best;       // [B]
+    int64_t *oldsum;     // [B]
+    int64_t *obj;        // [B]
+    int32_t *active;     // [B]
+    int32_t *improved;   // [B]
+    int32_t *accepted;   // [B]
+    int32_t *sweeps;     // [B]
+    int32_t *work;       // [W + 1][B]: step workers, then standalone ids
+    int32_t *kbud;       // [W + 1][B]: step budgets, then standalone budgets
+};
+
+static size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
+
+static pp_status plan_buffers(pp_instance *inst, int B, PlanBuffers *pb)
+{
+    const size_t n = (size_t)std::max(inst->n, 1);
+    const int W = inst->W;
+    size_t off[11], tot = 0;
+    const size_t sz[11] = {4 * n * B, 8 * n * B, 8 * (size_t)B, 8 * (size_t)B, 8 * (size_t)B,
+                           4 * (size_t)B, 4 * (size_t)B, 4 * (size_t)B, 4 * (size_t)B,
+                           4 * (size_t)(W + 1) * B, 4 * (size_t)(W + 1) * B};
+    for (int x = 0; x < 11; ++x) {
+        off[x] = tot;
+        tot += align_up(sz[x]);
+    }
+    pp_status s = ensure_scratch(inst->plan, tot);
+    if (s != PP_OK) return s;
+    char *base = reinterpret_cast<char *>(inst->plan.ptr);
+    pb->mask = reinterpret_cast<uint32_t *>(base + off[0]);
+    pb->profit = reinterpret_cast<int64_t *>(base + off[1]);
+    pb->best = reinterpret_cast<int64_t *>(base + off[2]);
+    pb->oldsum = reinterpret_cast<int64_t *>(base + off[3]);
+    pb->obj = reinterpret_cast<int64_t *>(base + off[4]);
+    pb->active = reinterpret_cast<int32_t *>(base + off[5]);
+    pb->improved = reinterpret_cast<int32_t *>(base + off[6]);
+    pb->accepted = reinterpret_cast<int32_t *>(base + off[7]);
+    pb->sweeps = reinterpret_cast<int32_t *>(base + off[8]);
+    pb->work = reinterpret_cast<int32_t *>(base + off[9]);
+    pb->kbud = reinterpret_cast<int32_t *>(base + off[10]);
+    return PP_OK;
+}
+
+static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t R,
+                           uint8_t *placement, int64_t *objective, pp_plan_stats *stats,
+                           cudaStream_t st)
+{
+    const int32_t n = inst->n, W = inst->W;
+    int launches = 0;
+    int64_t standalone_cells = 0;
+    int32_t maxk = 0;
+    int64_t sumk = 0;
+    for (int32_t m = 0; m < W; ++m) {
+        maxk = std::max(maxk, inst->h_budget[m]);
+        sumk += inst->h_budget[m];
+    }
+    DpGeom g;
+    if (!dp_geometry(inst, maxk, &g)) return fail(PP_EINVAL, "budget too large for the DP kernel");
+    const int B = std::max(S, W);
+    PlanBuffers pb;
+    pp_status s = plan_buffers(inst, B, &pb);
+    if (s != PP_OK) return s;
+    s = ensure_scratch(inst->plan_bits, (size_t)B * std::max(n, 1) * g.words * sizeof(uint32_t));
+    if (s != PP_OK) return s;
+    uint32_t *bits = reinterpret_cast<uint32_t *>(inst->plan_bits.ptr);
+
+    // ---- start orders -----------------------------------------------------
+    std::vector<int32_t> ord((size_t)S * W);
+    if (orders) {
+        for (int32_t x = 0; x < S; ++x) {
+            std::vector<int> seen(W, 0);
+            for (int32_t t = 0; t < W; ++t) {
+                int32_t h = orders[(size_t)x * W + t];
+                if (h < 0 || h >= W || seen[h]++) return fail(PP_EINVAL, "orders must be permutations of 0..W-1");
+            }
+        }
+        std::memcpy(ord.data(), orders, sizeof(int32_t) * ord.size());
+    } else {
+        for (int32_t x = 0; x < S; ++x)
+            std::iota(ord.begin() + (size_t)x * W, ord.begin() + (size_t)(x + 1) * W, 0);
+        if (S > 1) {
+            // standalone score of every worker: its DP optimum with no other holder
+            std::vector<int32_t> ids(W), kb(W);
+            std::iota(ids.begin(), ids.end(), 0);
+            for (int32_t m = 0; m < W; ++m) kb[m] = inst->h_budget[m];
+            int32_t *d_ids = pb.work + (size_t)W * B, *d_kb = pb.kbud + (size_t)W * B;
+            PP_CUDA(cudaMemcpyAsync(d_ids, ids.data(), 4 * W, cudaMemcpyHostToDevice, st));
+            PP_CUDA(cudaMemcpyAsync(d_kb, kb.data(), 4 * W, cudaMemcpyHostToDevice, st));
+            PP_CUDA(cudaMemsetAsync(pb.mask, 0, (size_t)4 * std::max(n, 1) * W, st));
+            if ((s = launch_marginals(inst, W, d_ids, pb.mask, false, nullptr, pb.profit, nullptr, st))) return s;
+            if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, g, pb.best, bits, st, maxk))) return s;
+            launches += 2;
+            std::vector<int64_t> score(W);
+            standalone_cells = (int64_t)n * sumk;
+            PP_CUDA(cudaMemcpyAsync(score.data(), pb.best, 8 * W, cudaMemcpyDeviceToHost, st));
+            PP_CUDA(cudaStreamSynchronize(st));
+            std::vector<int32_t> o(W);
+            std::iota(o.begin(), o.end(), 0);
+            std::stable_sort(o.begin(), o.end(), [&](int32_t x, int32_t y) { return score[x] > score[y]; });
+            std::copy(o.begin(), o.end(), ord.begin());
+            std::copy(o.rbegin(), o.rend(), ord.begin() + W);
+            for (int32_t x = 2; x < S; ++x) {
+                int32_t *q = ord.data() + (size_t)x * W;
+                uint64_t sm = (uint64_t)x;
+                for (int32_t i = W - 1; i >= 1; --i) {
+                    int32_t j = (int32_t)(splitmix64(sm) % (uint64_t)(i + 1));
+                    std::swap(q[i], q[j]);
+                }
+            }
+        }
+    }
+    if (stats && stats->orders_used) std::memcpy(stats->orders_used, ord.data(), sizeof(int32_t) * ord.size());
+
+    // ---- per-step worker / budget tables: work[t][s] = pi_s[t] -------------
+    std::vector<int32_t> hw((size_t)W * B, 0), hk((size_t)W * B, 0);
+    for (int32_t t = 0; t < W; ++t)
+        for (int32_t x = 0; x < S; ++x) {
+            int32_t h = ord[(size_t)x * W + t];
+            hw[(size_t)t * B + x] = h;
+            hk[(size_t)t * B + x] = inst->h_budget[h];
+        }
+    PP_CUDA(cudaMemcpyAsync(pb.work, hw.data(), 4 * hw.size(), cudaMemcpyHostToDevice, st));
+    PP_CUDA(cudaMemcpyAsync(pb.kbud, hk.data(), 4 * hk.size(), cudaMemcpyHostToDevice, st));
+    std::vector<int32_t> ones(S, 1);
+    PP_CUDA(cudaMemcpyAsync(pb.active, ones.data(), 4 * S, cudaMemcpyHostToDevice, st));
+    PP_CUDA(cudaMemsetAsync(pb.mask, 0, (size_t)4 * std::max(n, 1) * S, st));
+    PP_CUDA(cudaMemsetAsync(pb.accepted, 0, 4 * S, st));
+    PP_CUDA(cudaMemsetAsync(pb.sweeps, 0, 4 * S, st));
+
+    int dp_count = standalone_cells ? W : 0;
+    int64_t cells = standalone_cells;
+    auto step = [&](int t, int greedy) -> pp_status {
+        const int32_t *wk = pb.work + (size_t)t * B;
+        const int32_t *kb = pb.kbud + (size_t)t * B;
+        pp_status r;
+        if ((r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st))) return r;
+        if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, bits, st, maxk))) return r;
+        AcceptArgs a;
+        a.worker = wk;
+        a.best = pb.best;
+        a.oldsum = pb.oldsum;
+        a.active = pb.active;
+        a.improved = pb.improved;
+        a.accepted = pb.accepted;
+        a.mask = pb.mask;
+        a.greedy = greedy;
+        if ((r = launch_traceback(inst, S, bits, g, kb, nullptr, &a, st))) return r;
+        launches += 3;
+        return PP_OK;
+    };
+
+    // WorkerGreedy pass
+    for (int32_t t = 0; t < W; ++t)
+        if ((s = step(t, 1))) return s;
+    dp_count += S * W;
+    cells += (int64_t)S * n * sumk;
+
+    // coordinate refinement
+    std::vector<int32_t> act(S, 1);
+    for (int32_t r = 0; r < R; ++r) {
+        int nact = 0;
+        for (int32_t x = 0; x < S; ++x) nact += act[x] != 0;
+        if (nact == 0) break;
+        PP_CUDA(cudaMemsetAsync(pb.improved, 0, 4 * S, st));
+        for (int32_t t = 0; t < W; ++t)
+            if ((s = step(t, 0))) return s;
+        dp_count += nact * W;
+        cells += (int64_t)nact * n * sumk;
+        k_sweep_end<<<(S + 127) / 128, 128, 0, st>>>(S, pb.active, pb.improved, pb.sweeps);
+        PP_CUDA(cudaGetLastError());
+        launches += 1;
+        PP_CUDA(cudaMemcpyAsync(act.data(), pb.active, 4 * S, cudaMemcpyDeviceToHost, st));
+        PP_CUDA(cudaStreamSynchronize(st));
+    }
+
+    // objective of every candidate, argmax (ties to the lowest start)
+    if ((s = launch_objective(inst, S, pb.mask, nullptr, pb.obj, st))) return s;
+    launches += 1;
+    std::vector<int64_t> obj(S);
+    std::vector<int32_t> sw(S), acc(S);
+    PP_CUDA(cudaMemcpyAsync(obj.data(), pb.obj, 8 * S, cudaMemcpyDeviceToHost, st));
+    PP_CUDA(cudaMemcpyAsync(sw.data(), pb.sweeps, 4 * S, cudaMemcpyDeviceToHost, st));
+    PP_CUDA(cudaMemcpyAsync(acc.data(), pb.accepted, 4 * S, cudaMemcpyDeviceToHost, st));
+    PP_CUDA(cudaStreamSynchronize(st));
+    int32_t bs = 0;
+    for (int32_t x = 1; x < S; ++x)
+        if (obj[x] > obj[bs]) bs = x;
+    std::vector<uint32_t> mk(std::max(n, 1));
+    if (n > 0) {
+        PP_CUDA(cudaMemcpyAsync(mk.data(), pb.mask + (size_t)bs * n, 4 * (size_t)n, cudaMemcpyDeviceToHost, st));
+        PP_CUDA(cudaStreamSynchronize(st));
+    }
+    std::memset(placement, 0, (size_t)W * n);
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t b = inst->h_order[i];
+        uint32_t m = mk[i];
+        while (m) {
+            int h = __builtin_ctz(m);
+            m &= m - 1;
+            placement[(size_t)h * n + b] = 1;
+        }
+    }
+    *objective = obj[bs];
+    if (stats) {
+        if (stats->per_start_objective) std::copy(obj.begin(), obj.end(), stats->per_start_objective);
+        if (stats->per_start_sweeps) std::copy(sw.begin(), sw.end(), stats->per_start_sweeps);
+        if (stats->per_start_accepted) std::copy(acc.begin(), acc.end(), stats->per_start_accepted);
+        stats->best_start = bs;
+        stats->dp_count = dp_count;
+        stats->dp_cells = cells;
+        stats->kernel_launches = launches;
+    }
+    return PP_OK;
+}
+
+}  // namespace pp
+
+using namespace pp;
+
+extern "C" pp_status pp_plan_run(pp_instance *inst, int32_t n_starts, const int32_t *orders,
+                                 int32_t max_rounds, uint8_t *placement, int64_t *objective,
+                                 pp_plan_stats *stats, void *stream)
+{
+    if (!inst) return fail(PP_EINVAL, "null instance");
+    if (n_starts < 1) return fail(PP_EINVAL, "n_starts must be >= 1");
+    if (max_rounds < 0) return fail(PP_EINVAL, "max_rounds must be >= 0");
+    if (!objective || (inst->n > 0 && !placement)) return fail(PP_EINVAL, "null output pointer");
+    cudaStream_t st = (cudaStream_t)stream;
+    pp_status s = plan_impl(inst, n_starts, orders, max_rounds, placement, objective, stats, st);
+    if (s != PP_OK) return s;
+    return pp_instance_sync(inst, stream);
+}

@@ -1,0 +1,142 @@
+"""CPU checks of the C-ABI library: it loads, exports every declared entry
+point, and its host-side logic (validation, preorder, skip-row stack plan)
+is right.  No call here reaches a CUDA kernel."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2608_01655_gb300 import build as ppbuild
+from paper_2608_01655_gb300 import workloads as wl
+from tests import bruteforce as bf
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    ppbuild.build()
+    from paper_2608_01655_gb300 import binding
+    return binding
+
+
+def _declared():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            txt = open(os.path.join(ROOT, "include", f)).read()
+            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+            names |= set(re.findall(r"\b(pp_\w+)\s*\(", txt))
+    return names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    declared = _declared()
+    assert len(declared) >= 12
+    so = ctypes.CDLL(lib.LIB_PATH)
+    missing = [n for n in sorted(declared) if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def _create(lib, **kw):
+    inst = wl.random_small(np.random.default_rng(0), 6, 2, 0)
+    args = dict(n=inst.n, W=inst.W, parent=inst.parent, weight=inst.weight, demand=inst.demand,
+                recompute=inst.recompute, transfer=inst.transfer, mode=0, budget=inst.budget)
+    args.update(kw)
+    a = {k: (np.ascontiguousarray(v) if isinstance(v, np.ndarray) else v) for k, v in args.items()}
+    h = ctypes.c_void_p()
+    P = lambda x: x.ctypes.data_as(ctypes.c_void_p)
+    st = lib._lib.pp_instance_create(a["n"], a["W"], P(a["parent"].astype(np.int32)),
+                                     P(a["weight"].astype(np.int32)), P(a["demand"].astype(np.int64)),
+                                     P(a["recompute"].astype(np.int64)), P(a["transfer"].astype(np.int64)),
+                                     a["mode"], P(a["budget"].astype(np.int32)), None, ctypes.byref(h))
+    return st
+
+
+def test_create_validation_is_host_side(lib):
+    """Invalid instances are rejected before any CUDA call (Section III-A
+    feasibility data: a forest, weights >= 1, non-negative demand and costs)."""
+    assert _create(lib, parent=np.array([1, 2, 0, -1, -1, -1], np.int32)) == lib.PP_ENOTTREE
+    assert _create(lib, parent=np.array([0, -1, -1, -1, -1, -1], np.int32)) == lib.PP_ENOTTREE
+    assert _create(lib, parent=np.array([9, -1, -1, -1, -1, -1], np.int32)) == lib.PP_ENOTTREE
+    assert _create(lib, weight=np.array([1, 0, 1, 1, 1, 1], np.int32)) == lib.PP_EINVAL
+    dem = np.ones((2, 6), np.int64)
+    dem[1, 3] = -1
+    assert _create(lib, demand=dem) == lib.PP_EINVAL
+    assert _create(lib, W=0, budget=np.zeros(0, np.int32)) == lib.PP_EINVAL
+    assert _create(lib, W=33, budget=np.zeros(33, np.int32)) == lib.PP_EINVAL
+    assert _create(lib, mode=2) == lib.PP_EINVAL
+    assert _create(lib, budget=np.array([1, -1], np.int32)) == lib.PP_EINVAL
+    big = np.full((2, 6), 1 << 30, np.int64)       # 12 products of 2^60 > 2^62
+    assert _create(lib, demand=big, recompute=big) == lib.PP_EOVERFLOW
+    assert "2^62" in lib.last_error()
+
+
+def test_row_plan_preorder_matches_definition(lib):
+    """The library's preorder (independent of the oracle's) follows Section IV-A."""
+    rng = np.random.default_rng(2)
+    for trial in range(40):
+        inst = wl.random_small(rng, int(rng.integers(1, 60)), 1, 0)
+        order, nxt, skip, push, depth = lib.pp_row_plan(inst.parent)
+        assert list(order) == bf.preorder_positions(inst.parent)
+        size = {v: 1 for v in range(inst.n)}
+        for v in reversed(order):
+            if inst.parent[v] >= 0:
+                size[inst.parent[v]] += size[v]
+        assert list(nxt) == [i + size[v] for i, v in enumerate(order)]
+    with pytest.raises(lib.PPError):
+        lib.pp_row_plan(np.array([1, 0], np.int32))
+
+
+def _row_stack_dp(parent, weight, profit, k, plan):
+    """Eq. 9 swept exactly as the kernel does, driven by the row plan:
+    registers hold row i+1, the skip branch reads the code's source."""
+    order, nxt, skip, push, depth = plan
+    n = len(order)
+    cur = np.zeros(k + 1, np.int64)
+    stack = [None] * max(depth, 1)
+    for i in range(n - 1, -1, -1):
+        b = order[i]
+        s = cur.copy() if skip[i] == -1 else (np.zeros(k + 1, np.int64) if skip[i] == -2 else stack[skip[i]].copy())
+        new = s.copy()
+        w = weight[b]
+        for j in range(1, k + 1):
+            if j >= w:
+                t = profit[b] + cur[j - w]
+                if t > s[j]:
+                    new[j] = t
+        new[0] = 0
+        cur = new
+        if push[i] >= 0:
+            stack[push[i]] = cur.copy()
+    return int(cur[k])
+
+
+def test_row_plan_reproduces_the_dp(lib, oracle_lib):
+    """The skip-row stack plan feeds every row exactly the D[next(i)] of Eq. 9."""
+    rng = np.random.default_rng(3)
+    for trial in range(40):
+        n = int(rng.integers(1, 50))
+        inst = wl.random_small(rng, n, 1, 0, w_max=3)
+        profit = rng.integers(0, 20, size=n).astype(np.int64)
+        k = int(rng.integers(0, 12))
+        plan = lib.pp_row_plan(inst.parent)
+        best, _ = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, k)
+        assert _row_stack_dp(inst.parent, inst.weight, profit, k, plan) == best
+
+
+def test_row_plan_stack_depth_on_workloads(lib):
+    """The stack stays shallow on the workload trees (depth <= tree depth)."""
+    for cfg in (0, 1, 3):
+        inst = wl.make(cfg)
+        order, nxt, skip, push, depth = lib.pp_row_plan(inst.parent)
+        assert 1 <= depth <= inst.profile["max_depth"] + 1
+        # every stack read is preceded by a push to that level
+        live = set()
+        for i in range(inst.n - 1, -1, -1):
+            if skip[i] >= 0:
+                assert skip[i] in live
+            if push[i] >= 0:
+                live.add(push[i])

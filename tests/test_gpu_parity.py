@@ -1,0 +1,289 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Everything is integer, so the bar is bit-exact: profits, DP optima, chosen
+sets, objectives and whole plans must be identical.  Inputs come from the
+seeded generator only; expected values come from the oracle only.
+"""
+import numpy as np
+import pytest
+
+from paper_2608_01655_gb300 import workloads as wl
+from tests import bruteforce as bf
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def pp():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_01655_gb300 import build
+    build.build()
+    from paper_2608_01655_gb300 import binding
+    return binding
+
+
+def _dev(a, dtype):
+    return torch.from_numpy(np.ascontiguousarray(a).astype(dtype)).cuda()
+
+
+def _tree_instance(pp, parent, weight, W=1, mode=0, k=1):
+    n = len(parent)
+    inst = wl.Instance("t", n, W, np.asarray(parent, np.int32), np.asarray(weight, np.int32),
+                       np.ones((W, n), np.int64), np.ones((W, n), np.int64),
+                       np.ones((W, n), np.int64) if mode == 0 else np.ones((W, W, n), np.int64),
+                       mode, np.full(W, k, np.int32), 1, 1)
+    return pp.Instance.from_workload(inst)
+
+
+def _dp_batch(pp, ppi, profits, budgets, max_budget):
+    B, n = profits.shape
+    prof = _dev(profits, np.int64)
+    bud = _dev(budgets, np.int32)
+    best = torch.zeros(B, dtype=torch.int64, device="cuda")
+    bits = torch.zeros(max(pp.pp_dp_bits_size(ppi, B, max_budget) // 4, 1), dtype=torch.int32, device="cuda")
+    chosen = torch.zeros((B, n), dtype=torch.uint8, device="cuda")
+    pp.pp_tree_dp(ppi, prof, bud, max_budget, best, bits)
+    pp.pp_traceback(ppi, bits, bud, max_budget, chosen)
+    ppi.sync()
+    return best.cpu().numpy(), chosen.cpu().numpy()
+
+
+def _trees(rng):
+    """Small trees of many shapes: random forests (ids relabelled), chains,
+    stars, a binary tree and a single node."""
+    out = []
+    for _ in range(12):
+        out.append(wl.random_small(rng, int(rng.integers(1, 120)), 1, 0, w_max=4).parent)
+    out.append(np.arange(-1, 99, dtype=np.int32))                        # chain
+    out.append(np.full(77, -1, np.int32))                                 # star forest
+    out.append(np.array([-1] + [(v - 1) // 2 for v in range(1, 63)], np.int32))   # binary
+    out.append(np.array([-1], np.int32))
+    return out
+
+
+def test_tree_dp_and_traceback_small(pp, oracle_lib):
+    """Eq. 9 optimum and traced set, bit-exact, on many small trees and budgets
+    (k = 0, k inside, k above the total weight), with ties and negatives."""
+    rng = np.random.default_rng(100)
+    for parent in _trees(rng):
+        n = len(parent)
+        weight = rng.integers(1, 5, size=n).astype(np.int32)
+        ppi = _tree_instance(pp, parent, weight)
+        B = 6
+        profits = rng.integers(-3, 8, size=(B, n)).astype(np.int64)
+        profits[0] = np.maximum(profits[0], 0)
+        profits[1] = 0
+        tw = int(weight.sum())
+        budgets = np.array([0, 1, tw // 3, tw, tw + 7, int(rng.integers(0, tw + 1))], np.int32)
+        maxb = int(budgets.max())
+        best, chosen = _dp_batch(pp, ppi, profits, budgets, maxb)
+        for b in range(B):
+            ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+            assert best[b] == ob, (n, b)
+            np.testing.assert_array_equal(chosen[b], oc)
+        ppi.close()
+
+
+@pytest.mark.parametrize("n,wmax,kmax", [(700, 4, 1500), (3000, 4, 5000), (2500, 1, 2047),
+                                         (5000, 3, 9000), (1200, 1, 1061)])
+def test_tree_dp_multi_column_tiles(pp, oracle_lib, n, wmax, kmax):
+    """Budgets that span several columns per thread (C = 2..16) and ragged
+    tails (k not a multiple of 32), on deep and bushy trees."""
+    rng = np.random.default_rng(n + kmax)
+    inst = wl.random_small(rng, n, 1, 0, w_max=wmax)
+    parent = inst.parent
+    if n == 2500:                                     # deep: long chains with branching
+        parent = np.array([-1] + [v - 1 if rng.random() < 0.9 else int(rng.integers(v)) for v in range(1, n)],
+                          np.int32)
+    weight = inst.weight
+    ppi = _tree_instance(pp, parent, weight)
+    profits = rng.integers(0, 1000, size=(3, n)).astype(np.int64)
+    profits[1][rng.random(n) < 0.7] = 0
+    budgets = np.array([kmax, kmax - 13, kmax // 2 + 1], np.int32)
+    best, chosen = _dp_batch(pp, ppi, profits, budgets, kmax)
+    for b in range(3):
+        ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+        assert best[b] == ob
+        np.testing.assert_array_equal(chosen[b], oc)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_marginals_and_objective(pp, oracle_lib, mode):
+    """Eq. 10 / Eq. 7 marginals and Eq. 4 / Eq. 6 objectives, bit-exact."""
+    rng = np.random.default_rng(200 + mode)
+    for W in (1, 3, 7, 32):
+        inst = wl.random_small(rng, int(rng.integers(1, 300)), W, mode, demand_max=50)
+        prob = oracle_lib.Problem.from_instance(inst)
+        ppi = pp.Instance.from_workload(inst)
+        B = 5
+        pls = (rng.random((B, W, inst.n)) < rng.random((B, 1, 1))).astype(np.uint8)
+        masks = np.zeros((B, inst.n), np.uint32)
+        for m in range(W):
+            masks |= pls[:, m, :].astype(np.uint32) << np.uint32(m)
+        workers = rng.integers(0, W, size=B).astype(np.int32)
+        prof = torch.zeros((B, inst.n), dtype=torch.int64, device="cuda")
+        pp.pp_marginals(ppi, _dev(workers, np.int32), _dev(masks.view(np.int32), np.int32), prof)
+        obj = torch.zeros(B, dtype=torch.int64, device="cuda")
+        pp.pp_objective(ppi, _dev(pls, np.uint8), obj)
+        ppi.sync()
+        prof = prof.cpu().numpy()
+        obj = obj.cpu().numpy()
+        for b in range(B):
+            np.testing.assert_array_equal(prof[b], oracle_lib.marginal(prob, int(workers[b]), pls[b]))
+            assert obj[b] == oracle_lib.objective(prob, pls[b])
+        ppi.close()
+
+
+def _compare_plans(g, o):
+    np.testing.assert_array_equal(g.placement, o.placement)
+    assert g.objective == o.objective
+    assert g.best_start == o.best_start
+    np.testing.assert_array_equal(g.per_start_objective, o.per_start_objective)
+    np.testing.assert_array_equal(g.per_start_sweeps, o.per_start_sweeps)
+    np.testing.assert_array_equal(g.per_start_accepted, o.per_start_accepted)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_plan_small_random(pp, oracle_lib, mode):
+    """Algorithm 1 end to end on small random instances, explicit and default orders."""
+    rng = np.random.default_rng(300 + mode)
+    for trial in range(10):
+        W = int(rng.integers(1, 9))
+        inst = wl.random_small(rng, int(rng.integers(1, 200)), W, mode, k_max=60, w_max=3, demand_max=30)
+        prob = oracle_lib.Problem.from_instance(inst)
+        S = int(rng.integers(1, 5))
+        orders = wl.random_orders(W, S, seed=trial) if trial % 2 else None
+        with pp.Instance.from_workload(inst) as ppi:
+            g = pp.pp_plan_run(ppi, S, orders, 4)
+        o = oracle_lib.plan(prob, S, 4, orders=orders)
+        _compare_plans(g, o)
+        if orders is None:
+            np.testing.assert_array_equal(g.orders, oracle_lib.default_orders(prob, S))
+
+
+@pytest.mark.parametrize("cfg", [0, 1, 2])
+def test_plan_parity_workloads(pp, oracle_lib, cfg):
+    """Whole plans on the tiny, RAG and source-dependent workloads at full size:
+    placement, objective, per-start objectives, sweeps and accepts identical."""
+    inst = wl.make(cfg)
+    prob = oracle_lib.Problem.from_instance(inst)
+    with pp.Instance.from_workload(inst) as ppi:
+        g = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds)
+    o = oracle_lib.plan(prob, inst.starts, inst.rounds)
+    _compare_plans(g, o)
+    assert g.dp_cells == o.cells
+
+
+def _random_feasible_placement(rng, inst, frac):
+    """Parent-closed, within-budget placement grown top-down (a plausible
+    mid-refinement state to sample one update from)."""
+    order, nxt = oracle_lib_preorder(inst.parent)
+    pl = np.zeros((inst.W, inst.n), np.uint8)
+    for m in range(inst.W):
+        used = 0
+        take = rng.random(inst.n) < frac
+        for i, v in enumerate(order):
+            p = inst.parent[v]
+            if take[v] and (p < 0 or pl[m, p]) and used + inst.weight[v] <= inst.budget[m]:
+                pl[m, v] = 1
+                used += inst.weight[v]
+    return pl
+
+
+def oracle_lib_preorder(parent):
+    import oracle
+    return oracle.preorder(parent)
+
+
+@pytest.mark.parametrize("cfg", [3, 4])
+def test_single_update_full_size(pp, oracle_lib, cfg):
+    """One per-worker update (marginals -> DP -> traceback) at the full paper-
+    scale and stress sizes, against the oracle computing that one update."""
+    inst = wl.make(cfg)
+    prob = oracle_lib.Problem.from_instance(inst)
+    rng = np.random.default_rng(400 + cfg)
+    pl = _random_feasible_placement(rng, inst, 0.3)
+    h = int(rng.integers(inst.W))
+    masks = np.zeros(inst.n, np.uint32)
+    for m in range(inst.W):
+        masks |= pl[m].astype(np.uint32) << np.uint32(m)
+    with pp.Instance.from_workload(inst) as ppi:
+        prof = torch.zeros((1, inst.n), dtype=torch.int64, device="cuda")
+        pp.pp_marginals(ppi, _dev([h], np.int32), _dev(masks[None].view(np.int32), np.int32), prof)
+        k = int(inst.budget[h])
+        best = torch.zeros(1, dtype=torch.int64, device="cuda")
+        bits = torch.zeros(pp.pp_dp_bits_size(ppi, 1, k) // 4, dtype=torch.int32, device="cuda")
+        chosen = torch.zeros((1, inst.n), dtype=torch.uint8, device="cuda")
+        bud = _dev([k], np.int32)
+        pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
+        pp.pp_traceback(ppi, bits, bud, k, chosen)
+        ppi.sync()
+    ob, oprof, och = oracle_lib.worker_update(prob, h, pl)
+    np.testing.assert_array_equal(prof.cpu().numpy()[0], oprof)
+    assert int(best.item()) == ob
+    np.testing.assert_array_equal(chosen.cpu().numpy()[0], och)
+
+
+def test_plan_paper_scale_properties(pp, oracle_lib):
+    """The n=50,000 / 16-worker / 16-start plan the benchmark times: every
+    target prefix-complete and within budget, objective equal to the oracle's
+    evaluation of the returned placement, best-of-starts, and (for the returned
+    start, when it converged) no worker can strictly improve (Section IV-C)."""
+    inst = wl.make(3)
+    prob = oracle_lib.Problem.from_instance(inst)
+    with pp.Instance.from_workload(inst) as ppi:
+        g = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds)
+    for m in range(inst.W):
+        assert bf.is_parent_closed(inst.parent, g.placement[m])
+        assert int(inst.weight[g.placement[m].astype(bool)].sum()) <= inst.budget[m]
+    assert oracle_lib.objective(prob, g.placement) == g.objective
+    assert g.objective == g.per_start_objective.max()
+    assert np.all(g.per_start_sweeps <= inst.rounds)
+    if g.per_start_sweeps[g.best_start] < inst.rounds:
+        for h in range(inst.W):
+            best, p, _ = oracle_lib.worker_update(prob, h, g.placement)
+            assert best <= int(p[g.placement[h].astype(bool)].sum())
+
+
+def test_degenerate_instances(pp, oracle_lib):
+    """n = 0, W = 1, every budget 0, a single chunk."""
+    for n, W, k in [(0, 2, 5), (1, 1, 1), (5, 3, 0), (1, 32, 3)]:
+        rng = np.random.default_rng(n * 10 + W)
+        inst = wl.random_small(rng, n, W, 1, k_max=k) if n else wl.Instance(
+            "empty", 0, W, np.zeros(0, np.int32), np.zeros(0, np.int32), np.zeros((W, 0), np.int64),
+            np.zeros((W, 0), np.int64), np.zeros((W, W, 0), np.int64), 1, np.full(W, k, np.int32), 1, 1)
+        if k == 0:
+            inst.budget[:] = 0
+        with pp.Instance.from_workload(inst) as ppi:
+            g = pp.pp_plan_run(ppi, 2, None, 2)
+        assert g.placement.shape == (W, n)
+        if n == 0 or k == 0:
+            assert g.objective == 0 and g.placement.sum() == 0
+        else:
+            o = oracle_lib.plan(oracle_lib.Problem.from_instance(inst), 2, 2)
+            _compare_plans(g, o)
+
+
+def test_device_bounds_errors(pp):
+    """A budget above the declared bound and a worker id out of range are
+    reported through the status word, not by faulting."""
+    inst = wl.random_small(np.random.default_rng(7), 30, 3, 0)
+    with pp.Instance.from_workload(inst) as ppi:
+        prof = torch.ones((1, 30), dtype=torch.int64, device="cuda")
+        best = torch.zeros(1, dtype=torch.int64, device="cuda")
+        bits = torch.zeros(pp.pp_dp_bits_size(ppi, 1, 4) // 4, dtype=torch.int32, device="cuda")
+        pp.pp_tree_dp(ppi, prof, _dev([9], np.int32), 4, best, bits)
+        with pytest.raises(pp.PPError) as e:
+            ppi.sync()
+        assert e.value.status == pp.PP_EBOUNDS
+        ppi.sync()                                    # the word was cleared
+        out = torch.zeros((1, 30), dtype=torch.int64, device="cuda")
+        pp.pp_marginals(ppi, _dev([5], np.int32), torch.zeros((1, 30), dtype=torch.int32, device="cuda"), out)
+        with pytest.raises(pp.PPError) as e:
+            ppi.sync()
+        assert e.value.status == pp.PP_EBOUNDS
+        with pytest.raises(pp.PPError):
+            pp.pp_tree_dp(ppi, prof, _dev([1], np.int32), -1, best, bits)
