@@ -222,6 +222,17 @@ pp_status pp_plan_run(pp_instance *inst, int32_t n_starts, const int32_t *orders
                       int32_t max_rounds, uint8_t *placement, int64_t *objective,
                       pp_plan_stats *stats, void *stream);
 
+/*
+ * pp_test_inject -- testing hook for the failure path of the DP kernel's
+ * bounded waits; it makes no GPU fault.  kind 1: from the next launch on, the
+ * chain warp with index `value` (-1 = none, the default) stops publishing
+ * its ring counter, so the warp to its right waits until its time limit
+ * (0.5 s) runs out, every warp of the launch leaves its loop, and
+ * pp_instance_sync() reports PP_ETIMEOUT with the context still usable.
+ * Applies to the current device.  Errors: PP_EINVAL, PP_ECUDA.
+ */
+pp_status pp_test_inject(int32_t kind, int32_t value);
+
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);
 

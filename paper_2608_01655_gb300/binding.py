@@ -57,6 +57,7 @@ _SIGS = {
     "pp_traceback": [_P, _i32, _P, _P, _i32, _P, _P],
     "pp_objective": [_P, _i32, _P, _P, _P],
     "pp_plan_run": [_P, _i32, _P, _i32, _P, _P, ctypes.POINTER(PlanStats), _P],
+    "pp_test_inject": [_i32, _i32],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -224,3 +225,9 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                             ctypes.byref(st), _stream(stream)))
     return PlanResult(placement[:, :n].copy(), int(obj.value), int(st.best_start), per, sw, acc, used,
                       int(st.dp_count), int(st.dp_cells), int(st.kernel_launches))
+
+
+def pp_test_inject(kind: int, value: int):
+    """Testing hook: kind 1 makes chain warp `value` of later DP launches stop
+    publishing its ring counter (-1 restores normal operation)."""
+    _check(_lib.pp_test_inject(int(kind), int(value)))

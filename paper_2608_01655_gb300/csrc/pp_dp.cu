@@ -1,50 +1,416 @@
 // Exact capacity-k prefix-complete tree knapsack (Eq. 9, Theorem 1) and its
 // traceback (Algorithm 1, RootedDP).
 //
-// One CTA sweeps one DP instance.  Rows are preorder positions i = n-1..0;
-// the capacity axis is split across the CTA: thread t owns columns
-// t*C + c + 1 and keeps its part of row i+1 in registers.  Per row:
-//   skip  s_j = D[next(i)][j]: the registers (leaf, next(i) = i+1), zero
-//         (next(i) = n) or a saved row of the skip-row stack (shared memory
-//         for the top levels, instance scratch in global memory below them);
-//   take  t_j = p_i + D[i+1][j - w_i] for j >= w_i: row i+1 is also staged in
-//         shared memory (column-major per thread, conflict-free) so that the
-//         w_i-column shift can cross thread boundaries;
-//   D[i][j] = take ? t_j : s_j with take = (t_j > s_j), so the traceback
-//         yields the lexicographically smallest optimal preorder indicator;
-//   decision bits: one __ballot_sync per (warp, c) gives a 32-bit word,
-//         stored row-major at bits[i][warp*C + c].
-// Row metadata (p_i, w_i, skip/push codes) is staged through shared memory in
-// blocks of kMetaRows rows, prefetched one block ahead.
+//   D[i][0] = 0, D[n][j] = 0,
+//   D[i][j] = max{ D[next(i)][j], p_i + D[i+1][j - w_i] }   (take needs j >= w_i)
+//
+// Rows are preorder positions swept from n-1 down to 0, so row i needs row
+// i+1 and row next(i) > i.  Along the capacity axis column j needs only
+// column j of row next(i) and column j - w_i of row i+1: the dependency flows
+// from low to high columns.  Both kernels split the columns over threads,
+// each thread owning C consecutive columns in registers.
+//
+// k_tree_dp_wave (all chunk weights <= 4): one thread-block cluster of CL
+//   CTAs per DP, WPC warps per CTA, and no block-wide barrier in the row loop.
+//   Every warp sweeps its own columns row after row; warp g needs, for row i,
+//   the last w_i values of row i+1 of warp g-1, which that warp publishes
+//   into a ring in warp g's shared memory (DSMEM when g-1 is in the previous
+//   CTA of the cluster).  Ring counters are published with release stores
+//   every kPub rows and read with acquire loads; the consumer acknowledges
+//   slots so the producer never overwrites an unread one.  So warps form a
+//   wavefront, warp g lagging warp g-1 by a few rows.  Every wait is bounded
+//   in time and reports PP_ETIMEOUT through the status word.
+// k_tree_dp_flat (any weight): one CTA per DP, row i+1 staged in shared memory
+//   and one __syncthreads per row.
+//
+// Skip rows: next(i) = i+1 is the row just computed (registers), next(i) = n
+// is the zero row, and any other next(i) is the top of the skip-row stack,
+// which the wave kernel also keeps in registers (pushes store the new top to
+// shared memory, or to instance scratch below L_smem levels; pops reload it).
+//
+// Decision bits (take = strictly better, so the traceback returns the
+// lexicographically smallest optimal preorder indicator): one __ballot_sync
+// per (warp, c) gives the word ((item * P + g) * n + i) * C + c whose bit
+// `lane` is column (g * 32 + lane) * C + c + 1.
 #include <algorithm>
+#include <climits>
 
 #include "pp_internal.cuh"
 
 namespace pp {
 
+constexpr unsigned kFull = 0xffffffffu;
+
+// ===========================================================================
+// inline PTX helpers (cluster, DSMEM, acquire / release, timer)
+// ===========================================================================
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_nctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void st_cluster_s64(uint32_t addr, int64_t v)
+{
+    asm volatile("st.shared::cluster.s64 [%0], %1;" ::"r"(addr), "l"(v) : "memory");
+}
+__device__ __forceinline__ void st_release_cluster_u32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.release.cluster.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_release_cta_u32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_cluster_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint64_t global_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Testing hook (pp_test_inject): the chain warp with this index never
+// publishes its ring counter, so its right neighbour's bounded wait runs out.
+__device__ int32_t g_drop_publish_warp = -1;
+
+namespace wavecfg {
+constexpr int kRing = 64;                         // ring slots (rows), power of two
+constexpr int kPub = 8;                           // publish / acknowledge every kPub rows
+constexpr uint64_t kWaitLimitNs = 500ull * 1000 * 1000;   // one wait gives up after 0.5 s
+constexpr int64_t kNeg = LLONG_MIN / 2;           // D at a negative column: never taken
+}  // namespace wavecfg
+
+// Spin until the counter at `addr` (this CTA's shared memory, written by a
+// neighbour warp with release semantics) reaches `target`.  Warp-uniform.
+// Returns false if it waited longer than kWaitLimitNs or another wait of the
+// launch already timed out; the first to give up sets PP_ETIMEOUT.
+__device__ __forceinline__ bool wait_counter(uint32_t addr, uint32_t target, uint32_t &seen,
+                                          int32_t *status)
+{
+    uint64_t t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        uint32_t v = ld_acquire_cluster_u32(addr);
+        v = __shfl_sync(kFull, v, 0);
+        if (v >= target) {
+            seen = v;
+            return true;
+        }
+        if (it == 0) t0 = global_ns();
+        if ((it & 63) == 63) {
+            bool give_up = *(volatile int32_t *)status == PP_ETIMEOUT;
+            if (!give_up && global_ns() - t0 > wavecfg::kWaitLimitNs) {
+                give_up = true;
+                if ((threadIdx.x & 31) == 0) atomicExch(status, (int32_t)PP_ETIMEOUT);
+            }
+            if (__any_sync(kFull, give_up)) return false;
+            __nanosleep(64);
+        }
+    }
+}
+
+__host__ __device__ inline size_t wave_fixed_bytes(int WPC, int WMAX)
+{
+    size_t b = (size_t)WPC * wavecfg::kRing * WMAX * sizeof(int64_t) + 2 * (size_t)WPC * sizeof(uint32_t);
+    return (b + 15) & ~(size_t)15;
+}
+
+// take-branch base values sh[c] = D[i+1][col_c - W] for a static weight W:
+// own registers for c >= W, the left neighbour lane for c < W, and for lane 0
+// the boundary values bnd[q] = D[i+1][base - WMAX + q] of the previous warp.
+template <int C, int WMAX, int W>
+__device__ __forceinline__ void shift_by(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], int lane,
+                                         int64_t (&sh)[C])
+{
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+        if (c >= W) {
+            sh[c] = cur[c - W];
+        } else {
+            const int64_t v = __shfl_up_sync(kFull, cur[C - W + c], 1);
+            sh[c] = lane == 0 ? bnd[WMAX - W + c] : v;
+        }
+    }
+}
+
+template <int C, int WMAX>
+__device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], int lane,
+                                          int w, int64_t (&sh)[C])
+{
+    if (WMAX == 1) {
+        shift_by<C, WMAX, 1>(cur, bnd, lane, sh);
+    } else if (WMAX == 2) {
+        if (w == 1) shift_by<C, WMAX, 1>(cur, bnd, lane, sh);
+        else shift_by<C, WMAX, (WMAX >= 2 ? 2 : 1)>(cur, bnd, lane, sh);
+    } else {
+        switch (w) {
+        case 1: shift_by<C, WMAX, 1>(cur, bnd, lane, sh); break;
+        case 2: shift_by<C, WMAX, (WMAX >= 2 ? 2 : 1)>(cur, bnd, lane, sh); break;
+        case 3: shift_by<C, WMAX, (WMAX >= 3 ? 3 : 1)>(cur, bnd, lane, sh); break;
+        default: shift_by<C, WMAX, (WMAX >= 4 ? 4 : 1)>(cur, bnd, lane, sh); break;
+        }
+    }
+}
+
+// one row of cells: take = p + sh > s, D = take ? p + sh : s; ballot per c
+template <int C>
+__device__ __forceinline__ uint32_t row_cells(int64_t p, const int64_t (&sh)[C], const int64_t (&s)[C],
+                                              int lane, int64_t (&cur)[C])
+{
+    uint32_t word = 0;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+        const int64_t t = p + sh[c];
+        const bool take = t > s[c];
+        cur[c] = take ? t : s[c];
+        const uint32_t b = __ballot_sync(kFull, take);
+        word = lane == c ? b : word;
+    }
+    return word;
+}
+
+template <int C, int WMAX>
+__global__ void __launch_bounds__(512, 1)
+k_tree_dp_wave(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
+               const int32_t *__restrict__ wmeta, const int32_t *__restrict__ item_budget,
+               int32_t max_budget, const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
+               uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
+               int32_t *__restrict__ status)
+{
+    using namespace wavecfg;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int CL = (int)cluster_nctarank();
+    const int cr = (int)cluster_ctarank();
+    const int item = blockIdx.x / CL;
+    const int NT = blockDim.x;
+    const int WPC = NT >> 5;
+    const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int P = CL * WPC;
+    const int g = cr * WPC + wl;
+    const int kpad = P * 32 * C;
+
+    // uniform over the whole cluster: return before any DSMEM traffic
+    if (item_active && !item_active[item]) return;
+    const int32_t kreq = item_budget[item];
+    if (kreq < 0 || kreq > max_budget) {
+        if (cr == 0 && threadIdx.x == 0) {
+            atomicExch(status, (int32_t)PP_EBOUNDS);
+            best[item] = 0;
+        }
+        return;
+    }
+    const int k = kreq < kpad ? kreq : kpad;   // kpad covers min(max_budget, total weight)
+
+    int64_t *ring = reinterpret_cast<int64_t *>(smem);                          // [WPC][kRing][WMAX]
+    uint32_t *prog = reinterpret_cast<uint32_t *>(ring + (size_t)WPC * kRing * WMAX);   // [WPC]
+    uint32_t *ack = prog + WPC;                                                 // [WPC]
+    int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX));      // [L_smem][C][NT]
+    if (threadIdx.x < WPC) {
+        prog[threadIdx.x] = 0;
+        ack[threadIdx.x] = 0;
+    }
+    cluster_sync_all();     // every CTA initialised before any remote write
+
+    const bool has_prev = g > 0, has_next = g < P - 1;
+    const bool next_remote = has_next && wl == WPC - 1;
+    const bool prev_remote = has_prev && wl == 0;
+    uint32_t nx_ring = 0, nx_prog = 0, pv_ack = 0;
+    if (has_next) {
+        const int nw = next_remote ? 0 : wl + 1;
+        const uint32_t lr = smem_addr(ring + (size_t)nw * kRing * WMAX), lp = smem_addr(prog + nw);
+        nx_ring = next_remote ? map_to_rank(lr, cr + 1) : lr;
+        nx_prog = next_remote ? map_to_rank(lp, cr + 1) : lp;
+    }
+    if (has_prev) {
+        const uint32_t la = smem_addr(ack + (prev_remote ? WPC - 1 : wl - 1));
+        pv_ack = prev_remote ? map_to_rank(la, cr - 1) : la;
+    }
+    const uint32_t my_prog = smem_addr(prog + wl), my_ack = smem_addr(ack + wl);
+    const int64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
+    uint32_t prog_seen = 0, ack_seen = 0;
+    bool aborted = false;
+    const bool publish = g != g_drop_publish_warp;
+
+    const int64_t *Pp = profit + (size_t)item * n;
+    uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)n * C;
+    int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
+
+    int64_t cur[C], top[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+        cur[c] = 0;          // row n is the zero boundary
+        top[c] = 0;
+    }
+    // row metadata, 32 rows per warp register block, prefetched one block ahead
+    int64_t pb0 = 0, pb1 = 0;
+    int32_t mb0 = 0, mb1 = 0;
+    {
+        const int r0 = lane, r1 = 32 + lane;
+        if (r0 < n) { const int i = n - 1 - r0; pb0 = Pp[order ? order[i] : i]; mb0 = wmeta[i]; }
+        if (r1 < n) { const int i = n - 1 - r1; pb1 = Pp[order ? order[i] : i]; mb1 = wmeta[i]; }
+    }
+
+    for (int r = 0; r < n; ++r) {
+        const int rl = r & 31;
+        if (rl == 0 && r > 0) {
+            pb0 = pb1;
+            mb0 = mb1;
+            const int rn = r + 32 + lane;
+            if (rn < n) {
+                const int i = n - 1 - rn;
+                pb1 = Pp[order ? order[i] : i];
+                mb1 = wmeta[i];
+            }
+        }
+        const int64_t p = __shfl_sync(kFull, pb0, rl);
+        const int32_t m = __shfl_sync(kFull, mb0, rl);
+        const int i = n - 1 - r;
+        const int w = (m & 7) + 1;
+        const int kind = (m >> 3) & 3;
+
+        // boundary values D[i+1][base - WMAX + q] from the previous warp
+        int64_t bnd[WMAX];
+        if (has_prev) {
+#pragma unroll
+            for (int q = 0; q < WMAX; ++q) bnd[q] = 0;          // row n: zeros
+            if (r > 0) {
+                if (prog_seen < (uint32_t)r && !wait_counter(my_prog, (uint32_t)r, prog_seen, status)) {
+                    aborted = true;
+                    break;
+                }
+                if (lane == 0) {
+                    const int64_t *slot = my_ring + (size_t)((r - 1) & (kRing - 1)) * WMAX;
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q) bnd[q] = slot[q];
+                }
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < WMAX; ++q) bnd[q] = q == WMAX - 1 ? 0 : kNeg;   // columns 0, -1, ...
+        }
+
+        int64_t sh[C];
+        shift_row<C, WMAX>(cur, bnd, lane, w, sh);
+        int64_t s[C];
+#pragma unroll
+        for (int c = 0; c < C; ++c) s[c] = kind == kWaveCur ? cur[c] : (kind == kWaveTop ? top[c] : 0);
+        const uint32_t word = row_cells<C>(p, sh, s, lane, cur);
+        if (lane < C) Bw[(size_t)i * C + lane] = word;
+
+        // publish this row's last WMAX columns to the next warp
+        if (has_next) {
+            if (r + 2 > kRing && ack_seen < (uint32_t)(r + 2 - kRing) &&
+                !wait_counter(my_ack, (uint32_t)(r + 2 - kRing), ack_seen, status)) {
+                aborted = true;
+                break;
+            }
+            if (lane == 31) {
+                const uint32_t slot = nx_ring + (uint32_t)((r & (kRing - 1)) * WMAX * sizeof(int64_t));
+                if (next_remote) {
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q) st_cluster_s64(slot + q * 8, cur[C - WMAX + q]);
+                } else {
+                    int64_t *ls = ring + (size_t)(wl + 1) * kRing * WMAX + (size_t)(r & (kRing - 1)) * WMAX;
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q) ls[q] = cur[C - WMAX + q];
+                }
+                if (((r + 1) % kPub == 0 || r == n - 1) && publish) {
+                    if (next_remote) st_release_cluster_u32(nx_prog, (uint32_t)(r + 1));
+                    else st_release_cta_u32(nx_prog, (uint32_t)(r + 1));
+                }
+            }
+        }
+        // acknowledge consumed slots to the previous warp
+        if (has_prev && lane == 0 && ((r + 1) % kPub == 0 || r == n - 1)) {
+            if (prev_remote) st_release_cluster_u32(pv_ack, (uint32_t)(r + 1));
+            else st_release_cta_u32(pv_ack, (uint32_t)(r + 1));
+        }
+
+        // skip-row stack: push the new row (it becomes the top) or reload the top
+        if (m & kWavePush) {
+            const int lvl = (int)((uint32_t)m >> 16);
+#pragma unroll
+            for (int c = 0; c < C; ++c) {
+                top[c] = cur[c];
+                if (lvl < L_smem) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
+                else gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x] = cur[c];
+            }
+        } else if (m & kWaveReload) {
+            const int lvl = (int)((uint32_t)m >> 16);
+#pragma unroll
+            for (int c = 0; c < C; ++c)
+                top[c] = lvl < L_smem ? stk[((size_t)lvl * C + c) * NT + threadIdx.x]
+                                      : gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x];
+        }
+    }
+
+    if (!aborted) {
+        if (k == 0) {
+            if (g == 0 && lane == 0) best[item] = 0;
+        } else {
+            const int q = k - 1;
+            const int tt = q / C;
+            const int cc = q - tt * C;
+            int64_t v = cur[0];
+#pragma unroll
+            for (int c = 1; c < C; ++c) v = cc == c ? cur[c] : v;
+            if (g == (tt >> 5) && lane == (tt & 31)) best[item] = v;
+        }
+    }
+    cluster_sync_all();     // no CTA leaves while a neighbour may still write its shared memory
+}
+
+// ===========================================================================
+// General kernel (any chunk weight): one CTA, one barrier per row.
+// ===========================================================================
 constexpr int kMetaRows = 256;
 
-static size_t dp_smem_fixed(const DpGeom &g)
+static size_t flat_smem_fixed(int kpad)
 {
-    return 2 * (size_t)g.kpad * sizeof(int64_t) + 2 * kMetaRows * (sizeof(int64_t) + 2 * sizeof(int32_t));
+    return 2 * (size_t)kpad * sizeof(int64_t) + 2 * kMetaRows * (sizeof(int64_t) + 2 * sizeof(int32_t));
 }
 
 template <int C>
 __global__ void __launch_bounds__(1024, 1)
-k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
-          const int32_t *__restrict__ wpre, const int32_t *__restrict__ meta,
-          const int32_t *__restrict__ item_budget, int32_t max_budget,
-          const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
-          uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
-          int32_t *__restrict__ status)
+k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
+               const int32_t *__restrict__ wpre, const int32_t *__restrict__ meta,
+               const int32_t *__restrict__ item_budget, int32_t max_budget,
+               const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
+               uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
+               int32_t *__restrict__ status)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     const int T = blockDim.x;
     const int t = threadIdx.x;
     const int lane = t & 31, warp = t >> 5;
+    const int P = T >> 5;
     const int item = blockIdx.x;
     const int kpad = T * C;
-    const int words = kpad >> 5;
 
     if (item_active && !item_active[item]) return;
     const int32_t kreq = item_budget[item];
@@ -55,7 +421,7 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
         }
         return;
     }
-    const int k = kreq < kpad ? kreq : kpad;   // kpad covers min(max_budget, total weight)
+    const int k = kreq < kpad ? kreq : kpad;
 
     int64_t *srow = reinterpret_cast<int64_t *>(smem);          // [2][C][T]
     int64_t *sstk = srow + 2 * (size_t)kpad;                    // [L_smem][C][T]
@@ -63,18 +429,18 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
     int32_t *sw = reinterpret_cast<int32_t *>(sp + 2 * kMetaRows);
     int32_t *sm = sw + 2 * kMetaRows;
     int64_t *gst = gstack + (size_t)item * L_glob * kpad;
-    const int64_t *P = profit + (size_t)item * n;
-    uint32_t *B = bits + (size_t)item * n * words;
+    const int64_t *Pp = profit + (size_t)item * n;
+    uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)n * C;
 
-    int64_t cur[C];                      // D[i+1][t*C + c + 1]
+    int64_t cur[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) {
-        cur[c] = 0;                      // row n is the zero boundary
+        cur[c] = 0;
         srow[c * T + t] = 0;
     }
     for (int x = t; x < kMetaRows && x < n; x += T) {
         const int i = n - 1 - x;
-        sp[x] = P[order ? order[i] : i];
+        sp[x] = Pp[order ? order[i] : i];
         sw[x] = wpre[i];
         sm[x] = meta[i];
     }
@@ -85,11 +451,11 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
     for (int r = 0; r < n; ++r) {
         const int i = n - 1 - r;
         const int blk = r / kMetaRows, off = r - blk * kMetaRows, buf = (blk & 1) * kMetaRows;
-        if (off == 0) {                  // prefetch the next metadata block into registers
+        if (off == 0) {
             const int x = (blk + 1) * kMetaRows + t;
             if (t < kMetaRows && x < n) {
                 const int ii = n - 1 - x;
-                nx_p = P[order ? order[ii] : ii];
+                nx_p = Pp[order ? order[ii] : ii];
                 nx_w = wpre[ii];
                 nx_m = meta[ii];
             }
@@ -98,8 +464,8 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
         const int w = sw[buf + off];
         const int32_t m = sm[buf + off];
         const int skip = meta_skip(m), push = meta_push(m);
-        const int64_t *prev = srow + (r & 1) * kpad;            // D[i+1], column-major
-        int64_t *outr = srow + ((r + 1) & 1) * kpad;            // D[i]
+        const int64_t *prev = srow + (r & 1) * kpad;
+        int64_t *outr = srow + ((r + 1) & 1) * kpad;
         uint32_t myword = 0;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
@@ -108,8 +474,7 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
             else if (skip == kSkipZero) s = 0;
             else if (skip < L_smem) s = sstk[((size_t)skip * C + c) * T + t];
             else s = gst[((size_t)(skip - L_smem) * C + c) * T + t];
-            const int col = t * C + c + 1;
-            const int jj = col - w;
+            const int jj = t * C + c + 1 - w;
             bool take = false;
             int64_t v = s;
             if (jj >= 0) {
@@ -126,10 +491,10 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
             }
             cur[c] = v;
             outr[c * T + t] = v;
-            const uint32_t bw = __ballot_sync(0xffffffffu, take);
+            const uint32_t bw = __ballot_sync(kFull, take);
             if (lane == c) myword = bw;
         }
-        if (lane < C) B[(size_t)i * words + warp * C + lane] = myword;
+        if (lane < C) Bw[(size_t)i * C + lane] = myword;
         if (push >= 0) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
@@ -137,7 +502,7 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
                 else gst[((size_t)(push - L_smem) * C + c) * T + t] = cur[c];
             }
         }
-        if (off == kMetaRows - 1) {      // publish the prefetched block
+        if (off == kMetaRows - 1) {
             const int x = (blk + 1) * kMetaRows + t;
             const int nb = ((blk + 1) & 1) * kMetaRows;
             if (t < kMetaRows && x < n) {
@@ -160,23 +525,21 @@ k_tree_dp(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restri
     }
 }
 
-// ---------------------------------------------------------------------------
-// Traceback from (0, k): read the decision bit of (i, j); take -> mark b_i,
-// j -= w_i, i += 1; skip -> i = next(i).  Stops at i = n or j = 0 (no column
-// 0 bit is ever set).  One thread walks; the block first clears the output.
-// Planner mode (acc != nullptr): the update of worker h is accepted in the
-// greedy pass, or in refinement iff D[0][k] > sum of p_h over the current
+// ===========================================================================
+// Traceback from (0, k): take -> mark b_i, j -= w_i, i += 1; skip -> i =
+// next(i); stop at i = n or j = 0.  One thread walks; the block first clears
+// the output.  Planner mode (acc.mask != nullptr): the update is accepted in
+// the greedy pass, or in refinement iff D[0][k] > sum of p_h over the current
 // T_h (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
 // replaces bit h of the holder masks by the traced set.
-// ---------------------------------------------------------------------------
+// ===========================================================================
 __global__ void __launch_bounds__(256)
-k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int kpad,
+k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int P, int kpad,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
             const int32_t *__restrict__ wpre, const int32_t *__restrict__ next,
             uint8_t *__restrict__ chosen, AcceptArgs acc)
 {
     const int item = blockIdx.x;
-    const int words = kpad >> 5;
     uint32_t hbit = 0;
     uint32_t *M = nullptr;
     if (acc.mask) {
@@ -198,15 +561,15 @@ k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int kpad,
         acc.improved[item] = 1;
         acc.accepted[item] += 1;
     }
-    int32_t kq = item_budget[item];
+    const int32_t kq = item_budget[item];
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
-    const uint32_t *Bi = bits + (size_t)item * n * words;
+    const uint32_t *Bi = bits + (size_t)item * P * (size_t)n * C;
     int32_t i = 0;
     while (i < n && j > 0) {
         const int q = j - 1;
         const int tt = q / C, c = q - tt * C;
-        const uint32_t word = Bi[(size_t)i * words + (tt >> 5) * C + c];
+        const uint32_t word = Bi[((size_t)(tt >> 5) * n + i) * C + c];
         if ((word >> (tt & 31)) & 1u) {
             if (M) M[i] |= hbit;
             else chosen[(size_t)item * n + order[i]] = 1;
@@ -218,30 +581,128 @@ k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int kpad,
     }
 }
 
-template <int C>
-static pp_status launch_dp_c(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
-                             const int32_t *item_budget, int32_t max_budget,
-                             const int32_t *item_active, const DpGeom &g, int64_t *best,
-                             uint32_t *bits, cudaStream_t st)
+// ===========================================================================
+// geometry and launch
+// ===========================================================================
+template <int C, int WMAX>
+static const void *wave_kernel() { return (const void *)k_tree_dp_wave<C, WMAX>; }
+
+static const void *wave_kernel_for(int C, int WMAX)
 {
-    int dev_smem = 0;
-    PP_CUDA(cudaDeviceGetAttribute(&dev_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, inst->device));
-    const size_t fixed = dp_smem_fixed(g);
-    const size_t row_bytes = (size_t)g.kpad * sizeof(int64_t);
-    if (fixed > (size_t)dev_smem) return fail(PP_EINVAL, "budget too large for the DP kernel");
-    int L_smem = (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)dev_smem - fixed) / row_bytes);
-    int L_glob = inst->stack_depth - L_smem;
-    if (L_glob > 0) {
-        pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * row_bytes);
-        if (s != PP_OK) return s;
+#define PP_WAVE_CASE(CC, WW) if (C == CC && WMAX == WW) return wave_kernel<CC, WW>();
+    PP_WAVE_CASE(1, 1) PP_WAVE_CASE(2, 1) PP_WAVE_CASE(4, 1) PP_WAVE_CASE(8, 1) PP_WAVE_CASE(16, 1)
+    PP_WAVE_CASE(2, 2) PP_WAVE_CASE(4, 2) PP_WAVE_CASE(8, 2) PP_WAVE_CASE(16, 2)
+    PP_WAVE_CASE(4, 4) PP_WAVE_CASE(8, 4) PP_WAVE_CASE(16, 4)
+#undef PP_WAVE_CASE
+    return nullptr;
+}
+
+static int max_smem_optin(const pp_instance *inst)
+{
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, inst->device);
+    return v;
+}
+
+static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom *g)
+{
+    const int WMAX = inst->max_weight <= 1 ? 1 : (inst->max_weight <= 2 ? 2 : 4);
+    const int smem_max = max_smem_optin(inst);
+    int per_item = inst->sm_count / std::max(batch, 1);
+    per_item = std::max(1, std::min(8, per_item));
+    const int64_t max_cl = std::max<int64_t>(1, (k + 32 * WMAX - 1) / (32 * WMAX));
+    for (int CL = (int)std::min<int64_t>(per_item, max_cl); CL >= 1; --CL) {
+        const int64_t cols = (k + CL - 1) / CL;
+        int C = WMAX;
+        while ((cols + 32 * C - 1) / (32 * C) > 8 && C < 16) C *= 2;
+        const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
+        if (WPC > 16) continue;
+        const void *fn = wave_kernel_for(C, WMAX);
+        if (!fn) continue;
+        const size_t fixed = wave_fixed_bytes(WPC, WMAX);
+        const size_t level = (size_t)C * WPC * 32 * sizeof(int64_t);
+        if (fixed > (size_t)smem_max) continue;
+        const int L_smem = (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed) / level);
+        const size_t smem = fixed + (size_t)L_smem * level;
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(CL * std::max(batch, 1));
+        cfg.blockDim = dim3(WPC * 32);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int clusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            clusters = 0;
+        }
+        if (clusters < 1) continue;
+        if (clusters < batch && CL > 1) continue;       // prefer fewer SMs per DP to a second wave
+        g->wave = 1;
+        g->CL = CL;
+        g->WPC = WPC;
+        g->C = C;
+        g->WMAX = WMAX;
+        g->P = CL * WPC;
+        g->T = g->P * 32;
+        g->kpad = g->T * C;
+        g->words = g->kpad / 32;
+        g->L_smem = L_smem;
+        g->smem = smem;
+        return true;
     }
-    const size_t smem = fixed + (size_t)L_smem * row_bytes;
-    PP_CUDA(cudaFuncSetAttribute(k_tree_dp<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    k_tree_dp<C><<<batch, g.T, smem, st>>>(inst->n, profit, by_node ? inst->d_order : nullptr,
-                                            inst->d_wpre, inst->d_meta, item_budget, max_budget,
-                                            item_active, best, bits,
-                                            reinterpret_cast<int64_t *>(inst->stack.ptr), L_smem,
-                                            L_glob, inst->d_status);
+    return false;
+}
+
+bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int batch)
+{
+    if (max_budget < 0) return false;
+    int64_t k = max_budget;
+    if (k > inst->total_weight) k = inst->total_weight;   // larger budgets change nothing
+    if (k < 1) k = 1;
+    if (inst->max_weight <= 4 && inst->n > 0 && wave_geometry(inst, k, batch, g)) return true;
+    int C = 1;
+    while ((int64_t)C * 1024 < k) C *= 2;
+    if (C > 32) return false;
+    int T = (int)((k + C - 1) / C);
+    T = (T + 31) / 32 * 32;
+    if (T < 32) T = 32;
+    g->wave = 0;
+    g->CL = 1;
+    g->C = C;
+    g->T = T;
+    g->P = T / 32;
+    g->WPC = g->P;
+    g->kpad = T * C;
+    g->words = g->kpad / 32;
+    const size_t fixed = flat_smem_fixed(g->kpad);
+    const size_t row_bytes = (size_t)g->kpad * sizeof(int64_t);
+    const int smem_max = inst->n > 0 ? max_smem_optin(inst) : 0;
+    if (inst->n > 0 && fixed > (size_t)smem_max) return false;
+    g->L_smem = inst->n > 0 ? (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed) / row_bytes) : 0;
+    g->smem = fixed + (size_t)g->L_smem * row_bytes;
+    return true;
+}
+
+template <int C>
+static pp_status launch_flat_c(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
+                               const int32_t *item_budget, int32_t max_budget,
+                               const int32_t *item_active, const DpGeom &g, int64_t *best,
+                               uint32_t *bits, int64_t *gstack, int L_glob, cudaStream_t st)
+{
+    PP_CUDA(cudaFuncSetAttribute(k_tree_dp_flat<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem));
+    k_tree_dp_flat<C><<<batch, g.T, g.smem, st>>>(inst->n, profit, by_node ? inst->d_order : nullptr,
+                                                   inst->d_wpre, inst->d_meta, item_budget, max_budget,
+                                                   item_active, best, bits, gstack, g.L_smem, L_glob,
+                                                   inst->d_status);
     PP_CUDA(cudaGetLastError());
     return PP_OK;
 }
@@ -255,13 +716,45 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
         PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
         return PP_OK;
     }
+    const int L_glob = inst->stack_depth - g.L_smem;
+    if (L_glob > 0) {
+        pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
+        if (s != PP_OK) return s;
+    }
+    int64_t *gstack = reinterpret_cast<int64_t *>(inst->stack.ptr);
+    if (g.wave) {
+        const void *fn = wave_kernel_for(g.C, g.WMAX);
+        if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
+        PP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem));
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(g.CL * batch);
+        cfg.blockDim = dim3(g.WPC * 32);
+        cfg.dynamicSmemBytes = g.smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = g.CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int32_t n = inst->n;
+        const int32_t *order = by_node ? inst->d_order : nullptr;
+        const int32_t *wm = inst->d_wave;
+        int32_t L_smem = g.L_smem, Lg = L_glob;
+        int32_t *status = inst->d_status;
+        void *args[] = {&n, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
+                        (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status};
+        PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
+        return PP_OK;
+    }
     switch (g.C) {
-    case 1: return launch_dp_c<1>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
-    case 2: return launch_dp_c<2>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
-    case 4: return launch_dp_c<4>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
-    case 8: return launch_dp_c<8>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
-    case 16: return launch_dp_c<16>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
-    case 32: return launch_dp_c<32>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, st);
+    case 1: return launch_flat_c<1>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 2: return launch_flat_c<2>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 4: return launch_flat_c<4>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 8: return launch_flat_c<8>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 16: return launch_flat_c<16>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 32: return launch_flat_c<32>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
     default: return fail(PP_EINVAL, "unsupported DP geometry");
     }
 }
@@ -273,7 +766,7 @@ pp_status launch_traceback(pp_instance *inst, int batch, const uint32_t *bits, c
     if (batch <= 0 || inst->n == 0) return PP_OK;
     AcceptArgs a;
     if (acc) a = *acc;
-    k_traceback<<<batch, 256, 0, st>>>(inst->n, bits, g.C, g.kpad, item_budget, inst->d_order,
+    k_traceback<<<batch, 256, 0, st>>>(inst->n, bits, g.C, g.P, g.kpad, item_budget, inst->d_order,
                                        inst->d_wpre, inst->d_next, chosen, a);
     PP_CUDA(cudaGetLastError());
     return PP_OK;
@@ -286,7 +779,7 @@ using namespace pp;
 extern "C" size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_t max_budget)
 {
     DpGeom g;
-    if (!inst || batch <= 0 || !dp_geometry(inst, max_budget, &g)) return 0;
+    if (!inst || batch <= 0 || !dp_geometry(inst, max_budget, &g, batch)) return 0;
     return (size_t)batch * (size_t)inst->n * (size_t)g.words * sizeof(uint32_t);
 }
 
@@ -297,7 +790,7 @@ extern "C" pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t 
     if (!inst) return fail(PP_EINVAL, "null instance");
     if (batch < 0) return fail(PP_EINVAL, "batch must be >= 0");
     DpGeom g;
-    if (!dp_geometry(inst, max_budget, &g)) return fail(PP_EINVAL, "max_budget out of range");
+    if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
     if (batch == 0) return PP_OK;
     if (!budget || !best || (inst->n > 0 && (!profit || !bits)))
         return fail(PP_EINVAL, "null device pointer");
@@ -312,8 +805,15 @@ extern "C" pp_status pp_traceback(pp_instance *inst, int32_t batch, const uint32
     if (!inst) return fail(PP_EINVAL, "null instance");
     if (batch < 0) return fail(PP_EINVAL, "batch must be >= 0");
     DpGeom g;
-    if (!dp_geometry(inst, max_budget, &g)) return fail(PP_EINVAL, "max_budget out of range");
+    if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
     if (batch == 0 || inst->n == 0) return PP_OK;
     if (!bits || !budget || !chosen) return fail(PP_EINVAL, "null device pointer");
     return launch_traceback(inst, batch, bits, g, budget, chosen, nullptr, (cudaStream_t)stream);
+}
+
+extern "C" pp_status pp_test_inject(int32_t kind, int32_t value)
+{
+    if (kind != 1) return fail(PP_EINVAL, "unknown injection kind");
+    PP_CUDA(cudaMemcpyToSymbol(g_drop_publish_warp, &value, sizeof(value)));
+    return PP_OK;
 }

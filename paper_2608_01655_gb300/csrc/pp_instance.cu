@@ -1,6 +1,7 @@
 // Instance set-up: validation, preorder (Section IV-A), the DP's skip-row
 // stack plan, and the gain tables of Eq. 2-3 (requester-side) or Eq. 5
 // (source-dependent) computed on the device.
+#include <algorithm>
 #include <cstdio>
 #include <cstring>
 #include <new>
@@ -42,24 +43,6 @@ void free_scratch(Scratch &s)
     if (s.ptr) cudaFree(s.ptr);
     s.ptr = nullptr;
     s.bytes = 0;
-}
-
-bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g)
-{
-    if (max_budget < 0) return false;
-    int64_t k = max_budget;
-    if (k > inst->total_weight) k = inst->total_weight;   // larger budgets change nothing
-    int C = 1;
-    while ((int64_t)C * 1024 < k) C *= 2;
-    if (C > 32) return false;
-    int T = (int)((k + C - 1) / C);
-    T = (T + 31) / 32 * 32;
-    if (T < 32) T = 32;
-    g->C = C;
-    g->T = T;
-    g->kpad = T * C;
-    g->words = g->kpad / 32;
-    return true;
 }
 
 // ---------------------------------------------------------------------------
@@ -108,9 +91,11 @@ static bool build_preorder(int32_t n, const int32_t *parent, std::vector<int32_t
 
 // Skip-row stack plan: see the DP row metadata comment in pp_internal.cuh.
 static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vector<int32_t> &meta,
-                           int32_t *depth_out)
+                           int32_t *depth_out, const std::vector<int32_t> *wpre = nullptr,
+                           std::vector<int32_t> *wave = nullptr)
 {
     meta.assign(n, 0);
+    if (wave) wave->assign(n, 0);
     // last_reader[r] = smallest q with next(q) == r and q < r - 1 (stack reads only)
     std::vector<int32_t> last_reader(n + 1, -1);
     for (int32_t q = n - 1; q >= 0; --q) {
@@ -122,14 +107,17 @@ static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vec
     for (int32_t i = n - 1; i >= 0; --i) {
         int32_t r = next[i];
         int skip;
+        bool pop = false;
         if (r == i + 1) skip = kSkipCur;
         else if (r == n) skip = kSkipZero;
         else {
             skip = level[r];
-            if (skip < 0) return false;
+            // every stack read is of the top: the rows pushed after row r belong
+            // to the subtree of position i and were popped before i is reached
+            if (skip < 0 || skip != depth - 1) return false;
             if (last_reader[r] == i) {          // last reader: pop
                 --depth;
-                if (level[r] != depth) return false;
+                pop = true;
             }
         }
         int push = -1;
@@ -140,6 +128,19 @@ static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vec
             if (depth > kMaxStackLevels) return false;
         }
         meta[i] = meta_pack(skip, push);
+        if (wave) {
+            const int w = (*wpre)[i];
+            const int kind = skip == kSkipCur ? kWaveCur : (skip == kSkipZero ? kWaveZero : kWaveTop);
+            int flags = 0, lvl = 0;
+            if (push >= 0) {
+                flags = kWavePush;
+                lvl = push;
+            } else if (pop && depth > 0) {
+                flags = kWaveReload;                 // the level below becomes the top
+                lvl = depth - 1;
+            }
+            (*wave)[i] = wave_pack(w > 8 ? 8 : w, kind, flags, lvl);
+        }
     }
     *depth_out = maxd;
     return true;
@@ -208,6 +209,7 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     cudaFree(inst->d_next);
     cudaFree(inst->d_wpre);
     cudaFree(inst->d_meta);
+    cudaFree(inst->d_wave);
     cudaFree(inst->d_budget);
     cudaFree(inst->d_a);
     cudaFree(inst->d_delta);
@@ -264,14 +266,16 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     inst->mode = mode;
     if (!build_preorder(n, parent, inst->h_order, inst->h_next))
         return fail(PP_ENOTTREE, "parent array contains a cycle");
-    if (!build_row_meta(n, inst->h_next, inst->h_meta, &inst->stack_depth))
-        return fail(PP_EINVAL, "skip-row stack deeper than supported");
     inst->h_wpre.resize(n);
     inst->total_weight = 0;
+    inst->max_weight = 1;
     for (int32_t i = 0; i < n; ++i) {
         inst->h_wpre[i] = weight[inst->h_order[i]];
         inst->total_weight += weight[i];
+        inst->max_weight = std::max(inst->max_weight, weight[i]);
     }
+    if (!build_row_meta(n, inst->h_next, inst->h_meta, &inst->stack_depth, &inst->h_wpre, &inst->h_wave))
+        return fail(PP_EINVAL, "skip-row stack deeper than supported");
     inst->h_budget.assign(budget, budget + W);
 
     PP_CUDA(cudaGetDevice(&inst->device));
@@ -281,6 +285,7 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if ((s = upload(&inst->d_next, inst->h_next.data(), n, st))) return s;
     if ((s = upload(&inst->d_wpre, inst->h_wpre.data(), n, st))) return s;
     if ((s = upload(&inst->d_meta, inst->h_meta.data(), n, st))) return s;
+    if ((s = upload(&inst->d_wave, inst->h_wave.data(), n, st))) return s;
     if ((s = upload(&inst->d_budget, budget, W, st))) return s;
     PP_CUDA(cudaMalloc(&inst->d_status, sizeof(int32_t)));
     PP_CUDA(cudaMemsetAsync(inst->d_status, 0, sizeof(int32_t), st));

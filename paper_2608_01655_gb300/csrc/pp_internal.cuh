@@ -34,16 +34,38 @@ inline int32_t meta_pack(int skip, int push)
     return (int32_t)(((uint32_t)(push + 1) << 16) | (uint32_t)(skip + 2));
 }
 
+// Row metadata of the wavefront DP kernel: the skip-row stack top is kept in
+// registers (every stack read is of the top), so a row needs only: its weight,
+// where its skip row comes from, and whether it pushes (store the new row at
+// `level`, which becomes the top) or pops (reload the new top from `level`).
+// bits 0-2 weight-1 (weights <= 8), 3-4 kind, 5 reload, 6 push, 16-31 level.
+constexpr int kWaveCur = 0, kWaveZero = 1, kWaveTop = 2;
+constexpr int kWaveReload = 1 << 5, kWavePush = 1 << 6;
+inline int32_t wave_pack(int w, int kind, int flags, int level)
+{
+    return (int32_t)((uint32_t)(w - 1) | ((uint32_t)kind << 3) | (uint32_t)flags | ((uint32_t)level << 16));
+}
+
 // Column geometry of one DP launch: thread t of the chain owns columns
 // t*C + c + 1 (c = 0..C-1); column 0 is the boundary D[.][0] = 0.  Decision
 // bits of row i are kpad/32 words; word (t/32)*C + c holds bit (t%32) for the
 // column t*C + c + 1, i.e. one __ballot_sync per (warp, c).
 struct DpGeom {
     int C = 1;        // columns per thread
-    int T = 32;       // threads per chain
+    int T = 32;       // threads per chain (all CTAs)
     int kpad = 32;    // T * C columns
     int words = 1;    // decision words per row (kpad / 32)
+    int P = 1;        // warps per chain
+    int wave = 0;     // 1: wavefront kernel (cluster of CL CTAs x WPC warps)
+    int CL = 1;       // CTAs per chain (thread-block cluster)
+    int WPC = 1;      // warps per CTA
+    int WMAX = 1;     // largest chunk weight the wavefront kernel is built for
+    int L_smem = 0;   // skip-row stack levels held in shared memory
+    size_t smem = 0;  // dynamic shared memory per CTA
 };
+// Decision bits of every DP kernel: for chain warp g, preorder row i and
+// column offset c, word ((item * P + g) * n + i) * C + c holds bit `lane` for
+// column (g * 32 + lane) * C + c + 1.
 
 // Status word values written by kernels (same numbering as pp_status).
 constexpr int32_t kDevOk = PP_OK;
@@ -63,12 +85,14 @@ struct pp_instance {
     int sm_count = 0;
     int32_t stack_depth = 0;            // skip-row stack levels needed by the DP
     int64_t total_weight = 0;           // sum of chunk weights
-    std::vector<int32_t> h_order, h_next, h_budget, h_wpre, h_meta;
+    int32_t max_weight = 1;             // largest chunk weight
+    std::vector<int32_t> h_order, h_next, h_budget, h_wpre, h_meta, h_wave;
     // device tables, preorder-indexed unless noted
     int32_t *d_order = nullptr;         // [n] position -> node id
     int32_t *d_next = nullptr;          // [n]
     int32_t *d_wpre = nullptr;          // [n] chunk weight
     int32_t *d_meta = nullptr;          // [n] packed skip / push codes
+    int32_t *d_wave = nullptr;          // [n] wavefront-kernel row metadata
     int32_t *d_budget = nullptr;        // [W]
     int64_t *d_a = nullptr;             // mode 0: [W][n] a_m(b)       (Eq. 2)
     int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)
@@ -95,7 +119,7 @@ void free_scratch(Scratch &s);
 
 // DP launch geometry for a given largest budget (after clamping to the
 // instance's total weight).  Returns false when the budget is too large.
-bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g);
+bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int batch = 1);
 
 // Launchers used by both the ABI calls and the planner.
 //   prof_by_node: profits indexed by node id (ABI) instead of preorder

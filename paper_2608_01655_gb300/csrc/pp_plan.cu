@@ -91,13 +91,16 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         maxk = std::max(maxk, inst->h_budget[m]);
         sumk += inst->h_budget[m];
     }
-    DpGeom g;
-    if (!dp_geometry(inst, maxk, &g)) return fail(PP_EINVAL, "budget too large for the DP kernel");
+    // launch geometry of the start batch and of the standalone-score batch
+    DpGeom g, gw;
+    if (!dp_geometry(inst, maxk, &g, S) || !dp_geometry(inst, maxk, &gw, W))
+        return fail(PP_EINVAL, "budget too large for the DP kernel");
     const int B = std::max(S, W);
     PlanBuffers pb;
     pp_status s = plan_buffers(inst, B, &pb);
     if (s != PP_OK) return s;
-    s = ensure_scratch(inst->plan_bits, (size_t)B * std::max(n, 1) * g.words * sizeof(uint32_t));
+    const size_t nb = (size_t)std::max(n, 1);
+    s = ensure_scratch(inst->plan_bits, std::max((size_t)S * g.words, (size_t)W * gw.words) * nb * sizeof(uint32_t));
     if (s != PP_OK) return s;
     uint32_t *bits = reinterpret_cast<uint32_t *>(inst->plan_bits.ptr);
 
@@ -125,7 +128,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
             PP_CUDA(cudaMemcpyAsync(d_kb, kb.data(), 4 * W, cudaMemcpyHostToDevice, st));
             PP_CUDA(cudaMemsetAsync(pb.mask, 0, (size_t)4 * std::max(n, 1) * W, st));
             if ((s = launch_marginals(inst, W, d_ids, pb.mask, false, nullptr, pb.profit, nullptr, st))) return s;
-            if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, g, pb.best, bits, st, maxk))) return s;
+            if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, gw, pb.best, bits, st, maxk))) return s;
             launches += 2;
             std::vector<int64_t> score(W);
             standalone_cells = (int64_t)n * sumk;

@@ -287,3 +287,40 @@ def test_device_bounds_errors(pp):
         assert e.value.status == pp.PP_EBOUNDS
         with pytest.raises(pp.PPError):
             pp.pp_tree_dp(ppi, prof, _dev([1], np.int32), -1, best, bits)
+
+
+def test_flat_kernel_for_heavy_chunks(pp, oracle_lib):
+    """Chunk weights above 4 use the one-CTA kernel; same bits layout and traceback."""
+    rng = np.random.default_rng(500)
+    for n, wmax in [(400, 6), (1500, 9)]:
+        inst = wl.random_small(rng, n, 1, 0, w_max=wmax)
+        ppi = _tree_instance(pp, inst.parent, inst.weight)
+        profits = rng.integers(0, 50, size=(3, n)).astype(np.int64)
+        tw = int(inst.weight.sum())
+        budgets = np.array([tw // 4, tw // 2 + 3, 1500], np.int32)
+        best, chosen = _dp_batch(pp, ppi, profits, budgets, int(budgets.max()))
+        for b in range(3):
+            ob, oc = oracle_lib.rooted_dp(inst.parent, inst.weight, profits[b], int(budgets[b]))
+            assert best[b] == ob
+            np.testing.assert_array_equal(chosen[b], oc)
+
+
+def test_bounded_wait_reports_timeout(pp, oracle_lib):
+    """A chain warp that never publishes makes its neighbour's wait run out:
+    the launch ends with PP_ETIMEOUT (no fault), and the next launch is exact."""
+    rng = np.random.default_rng(600)
+    n, k = 600, 1024
+    inst = wl.random_small(rng, n, 1, 0)
+    ppi = _tree_instance(pp, inst.parent, inst.weight)
+    profits = rng.integers(0, 100, size=(1, n)).astype(np.int64)
+    try:
+        pp.pp_test_inject(1, 3)
+        with pytest.raises(pp.PPError) as e:
+            _dp_batch(pp, ppi, profits, np.array([k], np.int32), k)
+        assert e.value.status == pp.PP_ETIMEOUT
+    finally:
+        pp.pp_test_inject(1, -1)
+    best, chosen = _dp_batch(pp, ppi, profits, np.array([k], np.int32), k)
+    ob, oc = oracle_lib.rooted_dp(inst.parent, inst.weight, profits[0], k)
+    assert best[0] == ob
+    np.testing.assert_array_equal(chosen[0], oc)
