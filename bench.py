@@ -237,6 +237,9 @@ def run_native(args):
         total = float(t.item())
     value = world * cells_per_plan * args.steps / total
 
+    # ---- per-phase device time of one plan (events around every launch) ----
+    phased = pp.pp_plan_run(ppi, S, orders, R, time_phases=True)
+
     # ---- the dominant kernel, timed live: the plan's DP launch (S items) ----
     k = int(inst.budget.max())
     n = inst.n
@@ -351,6 +354,9 @@ def run_native(args):
                      "sweeps": res.per_start_sweeps.tolist(),
                      "step_ms": [round(1000 * t, 3) for t in times]},
             "marginals_launch_ms": 1000 * statistics.mean(mg_times),
+            "phase_ms": {"marginals": phased.phase_ms[0], "tree_dp": phased.phase_ms[1],
+                         "traceback_accept": phased.phase_ms[2]},
+            "dp_geometry": pp.pp_dp_geometry(ppi, S, k),
         }
         print(json.dumps(line), flush=True)
     ppi.close()

@@ -66,6 +66,9 @@ typedef struct {
     int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded) */
     int64_t dp_cells;              /* out: sum over executed DPs of n * k_h (Eq. 9 cells) */
     int32_t kernel_launches;       /* out: kernels launched by this call */
+    int32_t time_phases;           /* in: nonzero = time the phases below with CUDA events */
+    float phase_ms[3];             /* out (if time_phases): device time of the marginal,
+                                      tree-DP and traceback launches, summed over the plan */
 } pp_plan_stats;
 
 /*
@@ -124,6 +127,22 @@ pp_status pp_instance_preorder(const pp_instance *inst, int32_t *order, int32_t 
  */
 pp_status pp_row_plan(int32_t n, const int32_t *parent, int32_t *order, int32_t *next,
                       int32_t *skip_code, int32_t *push_level, int32_t *stack_depth);
+
+/*
+ * pp_row_plan_registers -- host-only: the per-row codes of the register-
+ * resident variant of the same row plan (the wavefront DP kernel keeps the
+ * top of the skip-row stack in registers; the zero row is the top of the
+ * empty stack).  code[i], i a preorder position (host [n] out):
+ *   bits 0-2   w_i - 1 (weights above 8 read as 8)
+ *   bits 3-4   0: the skip row is row i+1 (next(i) = i + 1); 2: the stack top
+ *   bit 5      after row i, reload the top from level `level`
+ *   bit 6      after row i, save row i at level `level`; it becomes the top
+ *   bit 7      after row i, the stack is empty: the top is the zero row
+ *   bits 16-31 level
+ * Errors: PP_EINVAL, PP_ENOTTREE.
+ */
+pp_status pp_row_plan_registers(int32_t n, const int32_t *parent, const int32_t *weight,
+                                int32_t *code);
 
 /*
  * pp_instance_sync -- synchronise `stream`, then read and clear the device
@@ -232,6 +251,24 @@ pp_status pp_plan_run(pp_instance *inst, int32_t n_starts, const int32_t *orders
  * Applies to the current device.  Errors: PP_EINVAL, PP_ECUDA.
  */
 pp_status pp_test_inject(int32_t kind, int32_t value);
+
+/*
+ * pp_dp_geometry -- the launch shape pp_tree_dp uses for `batch` items with
+ * budgets up to `max_budget` (host out[8]): wavefront kernel (1) or one-CTA
+ * kernel (0), CTAs per cluster, warps per CTA, columns per thread, warps per
+ * DP, skip-row stack levels in shared memory, shared memory bytes per CTA,
+ * padded column count.  Errors: PP_EINVAL.
+ */
+pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_budget, int32_t *out);
+
+/*
+ * pp_tune_dp -- process-wide override of the DP launch shape, for tuning
+ * sweeps: CTAs per cluster (1..8, 0 = automatic), columns per thread (power
+ * of two up to 16, 0 = automatic), force_flat != 0 selects the one-CTA kernel.
+ * Later pp_dp_bits_size / pp_tree_dp / pp_traceback / pp_plan_run calls use
+ * it, so set it before sizing workspaces.  Errors: PP_EINVAL.
+ */
+pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat);
 
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);

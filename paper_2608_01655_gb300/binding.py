@@ -43,7 +43,7 @@ class PPError(RuntimeError):
 class PlanStats(ctypes.Structure):
     _fields_ = [("per_start_objective", _P), ("per_start_sweeps", _P), ("per_start_accepted", _P),
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
-                ("kernel_launches", _i32)]
+                ("kernel_launches", _i32), ("time_phases", _i32), ("phase_ms", ctypes.c_float * 3)]
 
 
 _SIGS = {
@@ -51,6 +51,7 @@ _SIGS = {
     "pp_instance_destroy": [_P],
     "pp_instance_preorder": [_P, _P, _P, _P],
     "pp_row_plan": [_i32, _P, _P, _P, _P, _P, _P],
+    "pp_row_plan_registers": [_i32, _P, _P, _P],
     "pp_instance_sync": [_P, _P],
     "pp_marginals": [_P, _i32, _P, _P, _P, _P],
     "pp_tree_dp": [_P, _i32, _P, _P, _i32, _P, _P, _P],
@@ -58,6 +59,8 @@ _SIGS = {
     "pp_objective": [_P, _i32, _P, _P, _P],
     "pp_plan_run": [_P, _i32, _P, _i32, _P, _P, ctypes.POINTER(PlanStats), _P],
     "pp_test_inject": [_i32, _i32],
+    "pp_dp_geometry": [_P, _i32, _i32, _P],
+    "pp_tune_dp": [_i32, _i32, _i32],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -110,6 +113,16 @@ def pp_row_plan(parent):
     depth = _i32(0)
     _check(_lib.pp_row_plan(n, _host(parent), *[_host(o) for o in outs], ctypes.byref(depth)))
     return (*[o[:n] for o in outs], int(depth.value))
+
+
+def pp_row_plan_registers(parent, weight):
+    """Host-only per-row codes of the register-resident row plan (see the header)."""
+    parent = _np(parent, np.int32)
+    weight = _np(weight, np.int32)
+    n = parent.shape[0]
+    code = np.zeros(max(n, 1), np.int32)
+    _check(_lib.pp_row_plan_registers(n, _host(parent), _host(weight), _host(code)))
+    return code[:n]
 
 
 class Instance:
@@ -204,9 +217,11 @@ class PlanResult:
     dp_count: int
     dp_cells: int
     kernel_launches: int
+    phase_ms: tuple = ()
 
 
-def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None) -> PlanResult:
+def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
+                time_phases: bool = False) -> PlanResult:
     S, W, n = int(n_starts), inst.W, inst.n
     placement = np.zeros((W, max(n, 1)), np.uint8)
     obj = _i64(0)
@@ -214,7 +229,8 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     sw = np.zeros(S, np.int32)
     acc = np.zeros(S, np.int32)
     used = np.zeros((S, W), np.int32)
-    st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0)
+    st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0,
+                   int(bool(time_phases)))
     op = None
     if orders is not None:
         orders = _np(orders, np.int32)
@@ -224,10 +240,23 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     _check(_lib.pp_plan_run(inst.handle, S, op, int(max_rounds), _host(placement), ctypes.byref(obj),
                             ctypes.byref(st), _stream(stream)))
     return PlanResult(placement[:, :n].copy(), int(obj.value), int(st.best_start), per, sw, acc, used,
-                      int(st.dp_count), int(st.dp_cells), int(st.kernel_launches))
+                      int(st.dp_count), int(st.dp_cells), int(st.kernel_launches),
+                      tuple(float(x) for x in st.phase_ms) if time_phases else ())
 
 
 def pp_test_inject(kind: int, value: int):
     """Testing hook: kind 1 makes chain warp `value` of later DP launches stop
     publishing its ring counter (-1 restores normal operation)."""
     _check(_lib.pp_test_inject(int(kind), int(value)))
+
+
+def pp_dp_geometry(inst: Instance, batch: int, max_budget: int) -> dict:
+    out = np.zeros(8, np.int32)
+    _check(_lib.pp_dp_geometry(inst.handle, int(batch), int(max_budget), _host(out)))
+    keys = ["wave", "cluster_ctas", "warps_per_cta", "columns_per_thread", "warps_per_dp",
+            "stack_levels_smem", "smem_bytes", "kpad"]
+    return {k: int(v) for k, v in zip(keys, out)}
+
+
+def pp_tune_dp(cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: bool = False):
+    _check(_lib.pp_tune_dp(int(cluster_ctas), int(columns_per_thread), int(bool(force_flat))))

@@ -88,6 +88,36 @@ __device__ __forceinline__ uint32_t ld_acquire_cluster_u32(uint32_t addr)
     asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
     return v;
 }
+__device__ __forceinline__ void st_relaxed_cluster_u64(uint32_t addr, uint64_t v)
+{
+    asm volatile("st.relaxed.cluster.shared::cluster.u64 [%0], %1;" ::"r"(addr), "l"(v) : "memory");
+}
+__device__ __forceinline__ void st_relaxed_cluster_u32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.relaxed.cluster.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_relaxed_cluster_u64(uint32_t addr)
+{
+    uint64_t v;
+    asm volatile("ld.relaxed.cluster.shared::cta.u64 %0, [%1];" : "=l"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t ld_relaxed_cluster_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.relaxed.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_relaxed_cluster_u64_if(bool pred, uint32_t addr, uint64_t v)
+{
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %0, 0;\n\t"
+                 "@p st.relaxed.cluster.shared::cluster.u64 [%1], %2;\n\t}"
+                 ::"r"((uint32_t)pred), "r"(addr), "l"(v) : "memory");
+}
+__device__ __forceinline__ void ld_volatile_v2_u64(const uint64_t *p, uint64_t &a, uint64_t &b)
+{
+    asm volatile("ld.volatile.shared.v2.u64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(smem_addr(p)) : "memory");
+}
 __device__ __forceinline__ uint64_t global_ns()
 {
     uint64_t t;
@@ -106,21 +136,15 @@ constexpr uint64_t kWaitLimitNs = 500ull * 1000 * 1000;   // one wait gives up a
 constexpr int64_t kNeg = LLONG_MIN / 2;           // D at a negative column: never taken
 }  // namespace wavecfg
 
-// Spin until the counter at `addr` (this CTA's shared memory, written by a
-// neighbour warp with release semantics) reaches `target`.  Warp-uniform.
-// Returns false if it waited longer than kWaitLimitNs or another wait of the
-// launch already timed out; the first to give up sets PP_ETIMEOUT.
-__device__ __forceinline__ bool wait_counter(uint32_t addr, uint32_t target, uint32_t &seen,
-                                          int32_t *status)
+// Bounded spin (warp-uniform): `ready()` is re-evaluated until it holds.
+// Gives up after kWaitLimitNs, or as soon as another wait of the launch has
+// given up; the first to give up sets PP_ETIMEOUT.
+template <typename Ready>
+__device__ __forceinline__ bool spin_until(Ready ready, int32_t *status)
 {
     uint64_t t0 = 0;
     for (uint32_t it = 0;; ++it) {
-        uint32_t v = ld_acquire_cluster_u32(addr);
-        v = __shfl_sync(kFull, v, 0);
-        if (v >= target) {
-            seen = v;
-            return true;
-        }
+        if (__all_sync(kFull, ready())) return true;
         if (it == 0) t0 = global_ns();
         if ((it & 63) == 63) {
             bool give_up = *(volatile int32_t *)status == PP_ETIMEOUT;
@@ -129,20 +153,21 @@ __device__ __forceinline__ bool wait_counter(uint32_t addr, uint32_t target, uin
                 if ((threadIdx.x & 31) == 0) atomicExch(status, (int32_t)PP_ETIMEOUT);
             }
             if (__any_sync(kFull, give_up)) return false;
-            __nanosleep(64);
+            __nanosleep(32);
         }
     }
 }
 
 __host__ __device__ inline size_t wave_fixed_bytes(int WPC, int WMAX)
 {
-    size_t b = (size_t)WPC * wavecfg::kRing * WMAX * sizeof(int64_t) + 2 * (size_t)WPC * sizeof(uint32_t);
+    size_t b = (size_t)WPC * wavecfg::kRing * WMAX * sizeof(uint64_t) + (size_t)WPC * 32 * 16 +
+               (size_t)WPC * sizeof(uint32_t);
     return (b + 15) & ~(size_t)15;
 }
 
 // take-branch base values sh[c] = D[i+1][col_c - W] for a static weight W:
 // own registers for c >= W, the left neighbour lane for c < W, and for lane 0
-// the boundary values bnd[q] = D[i+1][base - WMAX + q] of the previous warp.
+// the boundary values bnd[q] = D[i+1][base - WMAX + 1 + q] of the previous warp.
 template <int C, int WMAX, int W>
 __device__ __forceinline__ void shift_by(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], int lane,
                                          int64_t (&sh)[C])
@@ -177,28 +202,27 @@ __device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t
     }
 }
 
-// one row of cells: take = p + sh > s, D = take ? p + sh : s; ballot per c
-template <int C>
-__device__ __forceinline__ uint32_t row_cells(int64_t p, const int64_t (&sh)[C], const int64_t (&s)[C],
-                                              int lane, int64_t (&cur)[C])
-{
-    uint32_t word = 0;
-#pragma unroll
-    for (int c = 0; c < C; ++c) {
-        const int64_t t = p + sh[c];
-        const bool take = t > s[c];
-        cur[c] = take ? t : s[c];
-        const uint32_t b = __ballot_sync(kFull, take);
-        word = lane == c ? b : word;
-    }
-    return word;
-}
+// Rows are swept in sub-blocks of kSub rows; the hand-off checks run once
+// per sub-block and the rows inside are unrolled.
+//
+// Hand-off between warp g-1 (producer) and warp g (consumer), fence-free:
+// for each row r the producer stores its last WMAX values of that row into
+// slot r % kRing of a ring in the consumer's shared memory, each as one
+// 64-bit word D | lap << 63 with lap = (r / kRing) % 2 (every D is in
+// [0, 2^62], so bit 63 is free).  A slot is self-validating: the consumer
+// re-reads the slots of a sub-block until every lap bit is the expected one.
+// The consumer reports the rows it has finished with a relaxed store into the
+// producer's shared memory, issued only after it used the values it read,
+// and the producer never writes a slot whose previous value is unread.
+constexpr int kSub = wavecfg::kPub;
+constexpr uint64_t kLapBit = 1ull << 63;
 
 template <int C, int WMAX>
 __global__ void __launch_bounds__(512, 1)
-k_tree_dp_wave(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
-               const int32_t *__restrict__ wmeta, const int32_t *__restrict__ item_budget,
-               int32_t max_budget, const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
+k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ profit,
+               const int32_t *__restrict__ order, const int32_t *__restrict__ wmeta,
+               const int32_t *__restrict__ item_budget, int32_t max_budget,
+               const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
                uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
                int32_t *__restrict__ status)
 {
@@ -226,147 +250,198 @@ k_tree_dp_wave(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
     }
     const int k = kreq < kpad ? kreq : kpad;   // kpad covers min(max_budget, total weight)
 
-    int64_t *ring = reinterpret_cast<int64_t *>(smem);                          // [WPC][kRing][WMAX]
-    uint32_t *prog = reinterpret_cast<uint32_t *>(ring + (size_t)WPC * kRing * WMAX);   // [WPC]
-    uint32_t *ack = prog + WPC;                                                 // [WPC]
-    int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX));      // [L_smem][C][NT]
-    if (threadIdx.x < WPC) {
-        prog[threadIdx.x] = 0;
-        ack[threadIdx.x] = 0;
-    }
+    uint64_t *ring = reinterpret_cast<uint64_t *>(smem);                           // [WPC][kRing][WMAX]
+    int4 *mstage = reinterpret_cast<int4 *>(ring + (size_t)WPC * kRing * WMAX);    // [WPC][32] (p, m)
+    uint32_t *ack = reinterpret_cast<uint32_t *>(mstage + (size_t)WPC * 32);       // [WPC]
+    int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX)); // [L_smem][C][NT]
+    for (int x = threadIdx.x; x < WPC * kRing * WMAX; x += NT) ring[x] = kLapBit;  // lap of row -1
+    if (threadIdx.x < WPC) ack[threadIdx.x] = 0;
     cluster_sync_all();     // every CTA initialised before any remote write
 
     const bool has_prev = g > 0, has_next = g < P - 1;
-    const bool next_remote = has_next && wl == WPC - 1;
     const bool prev_remote = has_prev && wl == 0;
-    uint32_t nx_ring = 0, nx_prog = 0, pv_ack = 0;
-    if (has_next) {
-        const int nw = next_remote ? 0 : wl + 1;
-        const uint32_t lr = smem_addr(ring + (size_t)nw * kRing * WMAX), lp = smem_addr(prog + nw);
-        nx_ring = next_remote ? map_to_rank(lr, cr + 1) : lr;
-        nx_prog = next_remote ? map_to_rank(lp, cr + 1) : lp;
-    }
+    // the next warp's ring through the cluster window (local or remote alike)
+    const uint32_t nx_ring = has_next ? map_to_rank(smem_addr(ring + (size_t)((wl + 1) % WPC) * kRing * WMAX),
+                                                    (uint32_t)(wl == WPC - 1 ? cr + 1 : cr)) : 0u;
+    uint32_t pv_ack = 0;
     if (has_prev) {
         const uint32_t la = smem_addr(ack + (prev_remote ? WPC - 1 : wl - 1));
         pv_ack = prev_remote ? map_to_rank(la, cr - 1) : la;
     }
-    const uint32_t my_prog = smem_addr(prog + wl), my_ack = smem_addr(ack + wl);
-    const int64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
-    uint32_t prog_seen = 0, ack_seen = 0;
+    const uint64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
+    int4 *my_meta = mstage + (size_t)wl * 32;
+    const uint32_t my_ack = smem_addr(ack + wl);
+    uint32_t ack_seen = 0;
     bool aborted = false;
-    const bool publish = g != g_drop_publish_warp;
+    const bool publish = has_next && lane == 31 && g != g_drop_publish_warp;   // this lane stores
 
     const int64_t *Pp = profit + (size_t)item * n;
-    uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)n * C;
+    uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
 
     int64_t cur[C], top[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) {
-        cur[c] = 0;          // row n is the zero boundary
+        cur[c] = 0;          // row n is the zero boundary, and the top of the empty stack
         top[c] = 0;
     }
-    // row metadata, 32 rows per warp register block, prefetched one block ahead
-    int64_t pb0 = 0, pb1 = 0;
-    int32_t mb0 = 0, mb1 = 0;
-    {
-        const int r0 = lane, r1 = 32 + lane;
-        if (r0 < n) { const int i = n - 1 - r0; pb0 = Pp[order ? order[i] : i]; mb0 = wmeta[i]; }
-        if (r1 < n) { const int i = n - 1 - r1; pb1 = Pp[order ? order[i] : i]; mb1 = wmeta[i]; }
-    }
-
-    for (int r = 0; r < n; ++r) {
-        const int rl = r & 31;
-        if (rl == 0 && r > 0) {
-            pb0 = pb1;
-            mb0 = mb1;
-            const int rn = r + 32 + lane;
-            if (rn < n) {
-                const int i = n - 1 - rn;
-                pb1 = Pp[order ? order[i] : i];
-                mb1 = wmeta[i];
-            }
+    // row metadata, 32 rows per block: lane l loads row blk*32 + l one block
+    // ahead and stages (p, m) in shared memory for the warp; rows past the
+    // last one are no-ops (p = -inf, skip = the row just computed), so every
+    // warp sweeps nblk * 32 rows
+    auto load_meta = [&](int r, int64_t &pv, int32_t &mv) {
+        if (r < n) {
+            const int i = n - 1 - r;
+            pv = Pp[order ? order[i] : i];
+            mv = wmeta[i];
+        } else {
+            pv = kNeg;
+            mv = 0;
         }
-        const int64_t p = __shfl_sync(kFull, pb0, rl);
-        const int32_t m = __shfl_sync(kFull, mb0, rl);
-        const int i = n - 1 - r;
-        const int w = (m & 7) + 1;
-        const int kind = (m >> 3) & 3;
-
-        // boundary values D[i+1][base - WMAX + q] from the previous warp
-        int64_t bnd[WMAX];
-        if (has_prev) {
+    };
+    int64_t pnext;
+    int32_t mnext;
+    load_meta(lane, pnext, mnext);
+    // boundary carried between sub-blocks: D[i+1][base - WMAX + 1 + q] of the
+    // previous warp for the first row of the next sub-block (row n: zeros)
+    int64_t carry[WMAX];
 #pragma unroll
-            for (int q = 0; q < WMAX; ++q) bnd[q] = 0;          // row n: zeros
-            if (r > 0) {
-                if (prog_seen < (uint32_t)r && !wait_counter(my_prog, (uint32_t)r, prog_seen, status)) {
+    for (int q = 0; q < WMAX; ++q) carry[q] = has_prev ? 0 : (q == WMAX - 1 ? 0 : kNeg);
+
+    for (int blk = 0; blk < nblk && !aborted; ++blk) {
+        __syncwarp();
+        my_meta[lane] = make_int4((int)(uint32_t)pnext, (int)(uint32_t)((uint64_t)pnext >> 32), mnext, 0);
+        const uint32_t stack_rows = __ballot_sync(kFull, (mnext & kWaveStackOps) != 0);   // bit = row of the block
+        __syncwarp();
+        load_meta((blk + 1) * 32 + lane, pnext, mnext);
+        uint32_t wbits[C];
+#pragma unroll
+        for (int c = 0; c < C; ++c) wbits[c] = 0;
+        for (int sb = 0; sb < 32 / kSub; ++sb) {
+            const int r0 = blk * 32 + sb * kSub;
+            // producer: slots r0..r0+kSub-1 last held rows r0-kRing.., which the
+            // consumer has finished reading once it reports row r0+kSub+1-kRing
+            if (has_next && r0 + kSub + 1 > kRing && ack_seen < (uint32_t)(r0 + kSub + 1 - kRing)) {
+                const uint32_t need = (uint32_t)(r0 + kSub + 1 - kRing);
+                if (!spin_until([&] { ack_seen = ld_relaxed_cluster_u32(my_ack); return ack_seen >= need; }, status)) {
                     aborted = true;
                     break;
                 }
-                if (lane == 0) {
-                    const int64_t *slot = my_ring + (size_t)((r - 1) & (kRing - 1)) * WMAX;
+            }
+            // consumer: rows r0..r0+kSub-1 of the previous warp, all with the
+            // lap bit of this pass over the ring
+            const uint64_t lap = (uint64_t)((r0 / kRing) & 1) << 63;
+            const uint64_t *sl = my_ring + (size_t)(r0 & (kRing - 1)) * WMAX;
+            uint64_t sv[WMAX == 1 ? kSub : 1];
+            if (has_prev) {
+                auto ready = [&] {
+                    uint64_t bad = 0;
+                    if (WMAX == 1) {
 #pragma unroll
-                    for (int q = 0; q < WMAX; ++q) bnd[q] = slot[q];
+                        for (int u = 0; u < kSub; u += 2) {
+                            uint64_t x, y;
+                            ld_volatile_v2_u64(sl + u, x, y);
+                            sv[u] = x;
+                            sv[u + 1] = y;
+                            bad |= (x ^ lap) | (y ^ lap);
+                        }
+                    } else {
+#pragma unroll
+                        for (int u = 0; u < kSub * WMAX; u += 2) {
+                            uint64_t x, y;
+                            ld_volatile_v2_u64(sl + u, x, y);
+                            bad |= (x ^ lap) | (y ^ lap);
+                        }
+                    }
+                    return (bad & kLapBit) == 0;
+                };
+                if (!spin_until(ready, status)) {
+                    aborted = true;
+                    break;
                 }
             }
-        } else {
+            const uint32_t mbase = 1u << (sb * kSub);
+            // one row of Eq. 9 for this warp's columns; STACK: the row may push or pop
+            auto row = [&](const int u, const bool STACK) {
+                const int r = r0 + u;
+                const int4 mm = my_meta[sb * kSub + u];
+                const int64_t p = (int64_t)(((uint64_t)(uint32_t)mm.y << 32) | (uint32_t)mm.x);
+                const int32_t m = mm.z;
+                // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
+                int64_t bnd[WMAX];
+                if (u == 0 || !has_prev) {
 #pragma unroll
-            for (int q = 0; q < WMAX; ++q) bnd[q] = q == WMAX - 1 ? 0 : kNeg;   // columns 0, -1, ...
-        }
-
-        int64_t sh[C];
-        shift_row<C, WMAX>(cur, bnd, lane, w, sh);
-        int64_t s[C];
-#pragma unroll
-        for (int c = 0; c < C; ++c) s[c] = kind == kWaveCur ? cur[c] : (kind == kWaveTop ? top[c] : 0);
-        const uint32_t word = row_cells<C>(p, sh, s, lane, cur);
-        if (lane < C) Bw[(size_t)i * C + lane] = word;
-
-        // publish this row's last WMAX columns to the next warp
-        if (has_next) {
-            if (r + 2 > kRing && ack_seen < (uint32_t)(r + 2 - kRing) &&
-                !wait_counter(my_ack, (uint32_t)(r + 2 - kRing), ack_seen, status)) {
-                aborted = true;
-                break;
-            }
-            if (lane == 31) {
-                const uint32_t slot = nx_ring + (uint32_t)((r & (kRing - 1)) * WMAX * sizeof(int64_t));
-                if (next_remote) {
-#pragma unroll
-                    for (int q = 0; q < WMAX; ++q) st_cluster_s64(slot + q * 8, cur[C - WMAX + q]);
+                    for (int q = 0; q < WMAX; ++q) bnd[q] = carry[q];
+                } else if (WMAX == 1) {
+                    bnd[0] = (int64_t)(sv[WMAX == 1 ? u - 1 : 0] & ~kLapBit);
                 } else {
-                    int64_t *ls = ring + (size_t)(wl + 1) * kRing * WMAX + (size_t)(r & (kRing - 1)) * WMAX;
 #pragma unroll
-                    for (int q = 0; q < WMAX; ++q) ls[q] = cur[C - WMAX + q];
+                    for (int q = 0; q < WMAX; ++q) bnd[q] = (int64_t)(sl[(u - 1) * WMAX + q] & ~kLapBit);
                 }
-                if (((r + 1) % kPub == 0 || r == n - 1) && publish) {
-                    if (next_remote) st_release_cluster_u32(nx_prog, (uint32_t)(r + 1));
-                    else st_release_cta_u32(nx_prog, (uint32_t)(r + 1));
+                int64_t sh[C];
+                shift_row<C, WMAX>(cur, bnd, lane, (m & 7) + 1, sh);
+                const bool from_cur = (m & (3 << 3)) == (kWaveCur << 3);
+                const uint32_t mrow = mbase << u;
+#pragma unroll
+                for (int c = 0; c < C; ++c) {
+                    const int64_t sk = from_cur ? cur[c] : top[c];
+                    const int64_t t = p + sh[c];
+                    const bool take = t > sk;
+                    cur[c] = take ? t : sk;
+                    if (take) wbits[c] |= mrow;
+                }
+                // hand this row's last WMAX columns to the next warp (lane 31 only)
+                {
+                    const uint32_t sa = nx_ring + (uint32_t)(((r & (kRing - 1)) * WMAX) * 8);
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q)
+                        st_relaxed_cluster_u64_if(publish, sa + q * 8, (uint64_t)cur[C - WMAX + q] | lap);
+                }
+                // skip-row stack: push (the new row becomes the top), reload or reset the top
+                if (STACK && (m & kWaveStackOps)) {
+                    const int lvl = (int)((uint32_t)m >> 16);
+                    if (m & kWavePush) {
+#pragma unroll
+                        for (int c = 0; c < C; ++c) {
+                            top[c] = cur[c];
+                            if (lvl < L_smem) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
+                            else gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x] = cur[c];
+                        }
+                    } else if (m & kWaveReload) {
+#pragma unroll
+                        for (int c = 0; c < C; ++c)
+                            top[c] = lvl < L_smem ? stk[((size_t)lvl * C + c) * NT + threadIdx.x]
+                                                  : gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x];
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < C; ++c) top[c] = 0;
+                    }
+                }
+            };
+            if (((stack_rows >> (sb * kSub)) & ((1u << kSub) - 1)) == 0) {
+#pragma unroll
+                for (int u = 0; u < kSub; ++u) row(u, false);       // no push or pop in these rows
+            } else {
+#pragma unroll
+                for (int u = 0; u < kSub; ++u) row(u, true);
+            }
+            if (has_prev) {
+                // the last row of this sub-block feeds the first row of the next one
+                if (WMAX == 1) {
+                    carry[0] = (int64_t)(sv[WMAX == 1 ? kSub - 1 : 0] & ~kLapBit);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q) carry[q] = (int64_t)(sl[(kSub - 1) * WMAX + q] & ~kLapBit);
+                }
+                // report the finished rows to the previous warp (values already used)
+                if (lane == 0) {
+                    if (prev_remote) st_relaxed_cluster_u32(pv_ack, (uint32_t)(r0 + kSub));
+                    else *(volatile uint32_t *)(ack + wl - 1) = (uint32_t)(r0 + kSub);
                 }
             }
         }
-        // acknowledge consumed slots to the previous warp
-        if (has_prev && lane == 0 && ((r + 1) % kPub == 0 || r == n - 1)) {
-            if (prev_remote) st_release_cluster_u32(pv_ack, (uint32_t)(r + 1));
-            else st_release_cta_u32(pv_ack, (uint32_t)(r + 1));
-        }
-
-        // skip-row stack: push the new row (it becomes the top) or reload the top
-        if (m & kWavePush) {
-            const int lvl = (int)((uint32_t)m >> 16);
 #pragma unroll
-            for (int c = 0; c < C; ++c) {
-                top[c] = cur[c];
-                if (lvl < L_smem) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
-                else gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x] = cur[c];
-            }
-        } else if (m & kWaveReload) {
-            const int lvl = (int)((uint32_t)m >> 16);
-#pragma unroll
-            for (int c = 0; c < C; ++c)
-                top[c] = lvl < L_smem ? stk[((size_t)lvl * C + c) * NT + threadIdx.x]
-                                      : gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x];
-        }
+        for (int c = 0; c < C; ++c) Bw[((size_t)blk * C + c) * 32] = wbits[c];
     }
 
     if (!aborted) {
@@ -430,7 +505,11 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
     int32_t *sm = sw + 2 * kMetaRows;
     int64_t *gst = gstack + (size_t)item * L_glob * kpad;
     const int64_t *Pp = profit + (size_t)item * n;
-    uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)n * C;
+    const int nblk = (n + 31) / 32;
+    uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)nblk * C * 32 + lane;
+    uint32_t wbits[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) wbits[c] = 0;
 
     int64_t cur[C];
 #pragma unroll
@@ -449,7 +528,6 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
     int64_t nx_p = 0;
     int32_t nx_w = 0, nx_m = 0;
     for (int r = 0; r < n; ++r) {
-        const int i = n - 1 - r;
         const int blk = r / kMetaRows, off = r - blk * kMetaRows, buf = (blk & 1) * kMetaRows;
         if (off == 0) {
             const int x = (blk + 1) * kMetaRows + t;
@@ -466,7 +544,7 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
         const int skip = meta_skip(m), push = meta_push(m);
         const int64_t *prev = srow + (r & 1) * kpad;
         int64_t *outr = srow + ((r + 1) & 1) * kpad;
-        uint32_t myword = 0;
+        const uint32_t mrow = 1u << (r & 31);
 #pragma unroll
         for (int c = 0; c < C; ++c) {
             int64_t s;
@@ -491,10 +569,15 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
             }
             cur[c] = v;
             outr[c * T + t] = v;
-            const uint32_t bw = __ballot_sync(kFull, take);
-            if (lane == c) myword = bw;
+            if (take) wbits[c] |= mrow;
         }
-        if (lane < C) Bw[(size_t)i * C + lane] = myword;
+        if ((r & 31) == 31 || r == n - 1) {
+#pragma unroll
+            for (int c = 0; c < C; ++c) {
+                Bw[((size_t)(r >> 5) * C + c) * 32] = wbits[c];
+                wbits[c] = 0;
+            }
+        }
         if (push >= 0) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
@@ -564,13 +647,15 @@ k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int P, int kpad
     const int32_t kq = item_budget[item];
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
-    const uint32_t *Bi = bits + (size_t)item * P * (size_t)n * C;
+    const int nblk = (n + 31) / 32;
+    const uint32_t *Bi = bits + (size_t)item * P * (size_t)nblk * C * 32;
     int32_t i = 0;
     while (i < n && j > 0) {
         const int q = j - 1;
         const int tt = q / C, c = q - tt * C;
-        const uint32_t word = Bi[((size_t)(tt >> 5) * n + i) * C + c];
-        if ((word >> (tt & 31)) & 1u) {
+        const int r = n - 1 - i;
+        const uint32_t word = Bi[(((size_t)(tt >> 5) * nblk + (r >> 5)) * C + c) * 32 + (tt & 31)];
+        if ((word >> (r & 31)) & 1u) {
             if (M) M[i] |= hbit;
             else chosen[(size_t)item * n + order[i]] = 1;
             j -= wpre[i];
@@ -590,9 +675,9 @@ static const void *wave_kernel() { return (const void *)k_tree_dp_wave<C, WMAX>;
 static const void *wave_kernel_for(int C, int WMAX)
 {
 #define PP_WAVE_CASE(CC, WW) if (C == CC && WMAX == WW) return wave_kernel<CC, WW>();
-    PP_WAVE_CASE(1, 1) PP_WAVE_CASE(2, 1) PP_WAVE_CASE(4, 1) PP_WAVE_CASE(8, 1) PP_WAVE_CASE(16, 1)
-    PP_WAVE_CASE(2, 2) PP_WAVE_CASE(4, 2) PP_WAVE_CASE(8, 2) PP_WAVE_CASE(16, 2)
-    PP_WAVE_CASE(4, 4) PP_WAVE_CASE(8, 4) PP_WAVE_CASE(16, 4)
+    PP_WAVE_CASE(1, 1) PP_WAVE_CASE(2, 1) PP_WAVE_CASE(4, 1) PP_WAVE_CASE(8, 1)
+    PP_WAVE_CASE(2, 2) PP_WAVE_CASE(4, 2) PP_WAVE_CASE(8, 2)
+    PP_WAVE_CASE(4, 4) PP_WAVE_CASE(8, 4)
 #undef PP_WAVE_CASE
     return nullptr;
 }
@@ -604,6 +689,9 @@ static int max_smem_optin(const pp_instance *inst)
     return v;
 }
 
+// Geometry overrides set by pp_tune_dp (0 = automatic).
+static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0;
+
 static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom *g)
 {
     const int WMAX = inst->max_weight <= 1 ? 1 : (inst->max_weight <= 2 ? 2 : 4);
@@ -611,10 +699,13 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     int per_item = inst->sm_count / std::max(batch, 1);
     per_item = std::max(1, std::min(8, per_item));
     const int64_t max_cl = std::max<int64_t>(1, (k + 32 * WMAX - 1) / (32 * WMAX));
-    for (int CL = (int)std::min<int64_t>(per_item, max_cl); CL >= 1; --CL) {
+    int cl_hi = (int)std::min<int64_t>(per_item, max_cl);
+    if (g_tune_cl > 0) cl_hi = std::min(g_tune_cl, 8);
+    for (int CL = cl_hi; CL >= 1; --CL) {
         const int64_t cols = (k + CL - 1) / CL;
         int C = WMAX;
-        while ((cols + 32 * C - 1) / (32 * C) > 8 && C < 16) C *= 2;
+        while ((cols + 32 * C - 1) / (32 * C) > 8 && C < 8) C *= 2;
+        if (g_tune_c > 0) C = std::max(std::min(g_tune_c, 8), WMAX);
         const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
         if (WPC > 16) continue;
         const void *fn = wave_kernel_for(C, WMAX);
@@ -668,7 +759,7 @@ bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int bat
     int64_t k = max_budget;
     if (k > inst->total_weight) k = inst->total_weight;   // larger budgets change nothing
     if (k < 1) k = 1;
-    if (inst->max_weight <= 4 && inst->n > 0 && wave_geometry(inst, k, batch, g)) return true;
+    if (inst->max_weight <= 4 && inst->n > 0 && !g_tune_flat && wave_geometry(inst, k, batch, g)) return true;
     int C = 1;
     while ((int64_t)C * 1024 < k) C *= 2;
     if (C > 32) return false;
@@ -739,11 +830,12 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         int32_t n = inst->n;
+        int32_t nblk = (n + 31) / 32;
         const int32_t *order = by_node ? inst->d_order : nullptr;
         const int32_t *wm = inst->d_wave;
         int32_t L_smem = g.L_smem, Lg = L_glob;
         int32_t *status = inst->d_status;
-        void *args[] = {&n, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
+        void *args[] = {&n, &nblk, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
                         (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status};
         PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
         return PP_OK;
@@ -780,7 +872,7 @@ extern "C" size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_
 {
     DpGeom g;
     if (!inst || batch <= 0 || !dp_geometry(inst, max_budget, &g, batch)) return 0;
-    return (size_t)batch * (size_t)inst->n * (size_t)g.words * sizeof(uint32_t);
+    return (size_t)batch * (size_t)((inst->n + 31) / 32 * 32) * (size_t)g.words * sizeof(uint32_t);
 }
 
 extern "C" pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t *profit,
@@ -815,5 +907,33 @@ extern "C" pp_status pp_test_inject(int32_t kind, int32_t value)
 {
     if (kind != 1) return fail(PP_EINVAL, "unknown injection kind");
     PP_CUDA(cudaMemcpyToSymbol(g_drop_publish_warp, &value, sizeof(value)));
+    return PP_OK;
+}
+
+extern "C" pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat)
+{
+    if (cluster_ctas < 0 || cluster_ctas > 8 || columns_per_thread < 0 || columns_per_thread > 16 ||
+        (columns_per_thread & (columns_per_thread - 1)) != 0)
+        return fail(PP_EINVAL, "cluster_ctas must be 0..8 and columns_per_thread 0 or a power of two <= 16");
+    g_tune_cl = cluster_ctas;
+    g_tune_c = columns_per_thread;
+    g_tune_flat = force_flat != 0;
+    return PP_OK;
+}
+
+extern "C" pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_budget,
+                                    int32_t *out)
+{
+    if (!inst || !out) return fail(PP_EINVAL, "null pointer");
+    DpGeom g;
+    if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
+    out[0] = g.wave;
+    out[1] = g.CL;
+    out[2] = g.WPC;
+    out[3] = g.C;
+    out[4] = g.P;
+    out[5] = g.L_smem;
+    out[6] = (int32_t)g.smem;
+    out[7] = g.kpad;
     return PP_OK;
 }

@@ -120,6 +120,7 @@ static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vec
                 pop = true;
             }
         }
+        const int32_t depth_read = depth;        // after any pop, before any push
         int push = -1;
         if (i >= 1 && last_reader[i] >= 0) {
             push = depth;
@@ -130,14 +131,18 @@ static bool build_row_meta(int32_t n, const std::vector<int32_t> &next, std::vec
         meta[i] = meta_pack(skip, push);
         if (wave) {
             const int w = (*wpre)[i];
-            const int kind = skip == kSkipCur ? kWaveCur : (skip == kSkipZero ? kWaveZero : kWaveTop);
+            // next(i) = n only happens with an empty stack, whose top is the zero row
+            if (skip == kSkipZero && depth_read != 0) return false;
+            const int kind = skip == kSkipCur ? kWaveCur : kWaveTop;
             int flags = 0, lvl = 0;
             if (push >= 0) {
                 flags = kWavePush;
                 lvl = push;
-            } else if (pop && depth > 0) {
+            } else if (pop && depth_read > 0) {
                 flags = kWaveReload;                 // the level below becomes the top
-                lvl = depth - 1;
+                lvl = depth_read - 1;
+            } else if (pop) {
+                flags = kWaveZeroTop;                // the stack emptied: top = zero row
             }
             (*wave)[i] = wave_pack(w > 8 ? 8 : w, kind, flags, lvl);
         }
@@ -373,6 +378,26 @@ extern "C" pp_status pp_row_plan(int32_t n, const int32_t *parent, int32_t *orde
         push_level[i] = meta_push(meta[i]);
     }
     if (stack_depth) *stack_depth = depth;
+    return PP_OK;
+}
+
+extern "C" pp_status pp_row_plan_registers(int32_t n, const int32_t *parent, const int32_t *weight,
+                                           int32_t *code)
+{
+    if (n < 0) return fail(PP_EINVAL, "n must be >= 0");
+    if (n > 0 && (!parent || !weight || !code)) return fail(PP_EINVAL, "null pointer");
+    for (int32_t v = 0; v < n; ++v) {
+        if (parent[v] < -1 || parent[v] >= n || parent[v] == v)
+            return fail(PP_ENOTTREE, "parent id out of range or self-parent at node " + std::to_string(v));
+        if (weight[v] < 1) return fail(PP_EINVAL, "chunk weight must be >= 1");
+    }
+    std::vector<int32_t> o, nx, meta, wave, wpre(n);
+    if (!build_preorder(n, parent, o, nx)) return fail(PP_ENOTTREE, "parent array contains a cycle");
+    for (int32_t i = 0; i < n; ++i) wpre[i] = weight[o[i]];
+    int32_t depth = 0;
+    if (!build_row_meta(n, nx, meta, &depth, &wpre, &wave))
+        return fail(PP_EINVAL, "skip-row stack deeper than supported");
+    for (int32_t i = 0; i < n; ++i) code[i] = wave[i];
     return PP_OK;
 }
 

@@ -35,12 +35,16 @@ inline int32_t meta_pack(int skip, int push)
 }
 
 // Row metadata of the wavefront DP kernel: the skip-row stack top is kept in
-// registers (every stack read is of the top), so a row needs only: its weight,
-// where its skip row comes from, and whether it pushes (store the new row at
-// `level`, which becomes the top) or pops (reload the new top from `level`).
-// bits 0-2 weight-1 (weights <= 8), 3-4 kind, 5 reload, 6 push, 16-31 level.
-constexpr int kWaveCur = 0, kWaveZero = 1, kWaveTop = 2;
-constexpr int kWaveReload = 1 << 5, kWavePush = 1 << 6;
+// registers (every stack read is of the top, and the zero row D[n][.] is the
+// top of the empty stack), so a row needs only: its weight, whether its skip
+// row is the row just computed (next(i) = i + 1) or the top, and whether it
+// pushes (store the new row at `level`; it becomes the top) or pops (reload
+// the new top from `level`, or reset it to the zero row when the stack empties).
+// bits 0-2 weight-1 (weights <= 8), 3-4 kind, 5 reload, 6 push, 7 zero top,
+// 16-31 level.
+constexpr int kWaveCur = 0, kWaveTop = 2;
+constexpr int kWaveReload = 1 << 5, kWavePush = 1 << 6, kWaveZeroTop = 1 << 7;
+constexpr int kWaveStackOps = kWaveReload | kWavePush | kWaveZeroTop;
 inline int32_t wave_pack(int w, int kind, int flags, int level)
 {
     return (int32_t)((uint32_t)(w - 1) | ((uint32_t)kind << 3) | (uint32_t)flags | ((uint32_t)level << 16));
@@ -63,9 +67,12 @@ struct DpGeom {
     int L_smem = 0;   // skip-row stack levels held in shared memory
     size_t smem = 0;  // dynamic shared memory per CTA
 };
-// Decision bits of every DP kernel: for chain warp g, preorder row i and
-// column offset c, word ((item * P + g) * n + i) * C + c holds bit `lane` for
-// column (g * 32 + lane) * C + c + 1.
+// Decision bits of every DP kernel, packed by each thread over blocks of 32
+// rows in sweep order (row r = n - 1 - i, block r / 32, bit r % 32): for chain
+// warp g, lane and column offset c, the word
+//   (((item * P + g) * nblk + r / 32) * C + c) * 32 + lane
+// holds the take decisions of column (g * 32 + lane) * C + c + 1, with
+// nblk = ceil(n / 32).
 
 // Status word values written by kernels (same numbering as pp_status).
 constexpr int32_t kDevOk = PP_OK;

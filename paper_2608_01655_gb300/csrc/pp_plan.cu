@@ -99,7 +99,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
     PlanBuffers pb;
     pp_status s = plan_buffers(inst, B, &pb);
     if (s != PP_OK) return s;
-    const size_t nb = (size_t)std::max(n, 1);
+    const size_t nb = (size_t)std::max((n + 31) / 32 * 32, 32);
     s = ensure_scratch(inst->plan_bits, std::max((size_t)S * g.words, (size_t)W * gw.words) * nb * sizeof(uint32_t));
     if (s != PP_OK) return s;
     uint32_t *bits = reinterpret_cast<uint32_t *>(inst->plan_bits.ptr);
@@ -169,12 +169,26 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
 
     int dp_count = standalone_cells ? W : 0;
     int64_t cells = standalone_cells;
+    // optional per-phase timing: events around every launch, read once at the end
+    const bool timing = stats && stats->time_phases;
+    std::vector<cudaEvent_t> ev;
+    auto mark = [&]() -> pp_status {
+        if (!timing) return PP_OK;
+        cudaEvent_t e;
+        PP_CUDA(cudaEventCreate(&e));
+        PP_CUDA(cudaEventRecord(e, st));
+        ev.push_back(e);
+        return PP_OK;
+    };
     auto step = [&](int t, int greedy) -> pp_status {
         const int32_t *wk = pb.work + (size_t)t * B;
         const int32_t *kb = pb.kbud + (size_t)t * B;
         pp_status r;
+        if ((r = mark())) return r;
         if ((r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st))) return r;
+        if ((r = mark())) return r;
         if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, bits, st, maxk))) return r;
+        if ((r = mark())) return r;
         AcceptArgs a;
         a.worker = wk;
         a.best = pb.best;
@@ -185,6 +199,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         a.mask = pb.mask;
         a.greedy = greedy;
         if ((r = launch_traceback(inst, S, bits, g, kb, nullptr, &a, st))) return r;
+        if ((r = mark())) return r;
         launches += 3;
         return PP_OK;
     };
@@ -249,7 +264,18 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         stats->dp_count = dp_count;
         stats->dp_cells = cells;
         stats->kernel_launches = launches;
+        stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
+        for (size_t x = 0; x + 3 < ev.size(); x += 4) {
+            float a = 0.f, b = 0.f, c = 0.f;
+            cudaEventElapsedTime(&a, ev[x], ev[x + 1]);
+            cudaEventElapsedTime(&b, ev[x + 1], ev[x + 2]);
+            cudaEventElapsedTime(&c, ev[x + 2], ev[x + 3]);
+            stats->phase_ms[0] += a;
+            stats->phase_ms[1] += b;
+            stats->phase_ms[2] += c;
+        }
     }
+    for (cudaEvent_t e : ev) cudaEventDestroy(e);
     return PP_OK;
 }
 

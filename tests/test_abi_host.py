@@ -140,3 +140,48 @@ def test_row_plan_stack_depth_on_workloads(lib):
                 assert skip[i] in live
             if push[i] >= 0:
                 live.add(push[i])
+
+
+def _register_dp(parent, weight, profit, k, order, code):
+    """Eq. 9 swept with the register-resident plan: `cur` is row i+1, `top`
+    the stack top (zero row when empty), saved levels in a list."""
+    n = len(order)
+    cur = np.zeros(k + 1, np.int64)
+    top = np.zeros(k + 1, np.int64)
+    levels = {}
+    for i in range(n - 1, -1, -1):
+        c = int(code[i])
+        w = (c & 7) + 1
+        kind = (c >> 3) & 3
+        assert w == min(int(weight[order[i]]), 8)
+        s = cur.copy() if kind == 0 else top.copy()
+        assert kind in (0, 2)
+        new = s.copy()
+        for j in range(1, k + 1):
+            if j >= w and profit[order[i]] + cur[j - w] > s[j]:
+                new[j] = profit[order[i]] + cur[j - w]
+        cur = new
+        lvl = (c >> 16) & 0xFFFF
+        if c & (1 << 6):
+            levels[lvl] = cur.copy()
+            top = cur.copy()
+        elif c & (1 << 5):
+            top = levels[lvl].copy()
+        elif c & (1 << 7):
+            top = np.zeros(k + 1, np.int64)
+    return int(cur[k])
+
+
+def test_register_row_plan_reproduces_the_dp(lib, oracle_lib):
+    """The register-resident plan (stack top in registers, zero row as the
+    empty stack's top) feeds every row the D[next(i)] of Eq. 9."""
+    rng = np.random.default_rng(4)
+    for trial in range(60):
+        n = int(rng.integers(1, 60))
+        inst = wl.random_small(rng, n, 1, 0, w_max=3)
+        profit = rng.integers(0, 20, size=n).astype(np.int64)
+        k = int(rng.integers(0, 14))
+        order, *_ = lib.pp_row_plan(inst.parent)
+        code = lib.pp_row_plan_registers(inst.parent, inst.weight)
+        best, _ = oracle_lib.rooted_dp(inst.parent, inst.weight, profit, k)
+        assert _register_dp(inst.parent, inst.weight, profit, k, order, code) == best, trial
