@@ -196,6 +196,35 @@ pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t *profit,
                      uint32_t *bits, void *stream);
 
 /*
+ * pp_tree_dp_noalloc -- pp_tree_dp for callers that must not allocate device
+ * memory while they plan.  The paper has no counterpart: it is a library
+ * convenience.  pp_tree_dp may call cudaMalloc on first use, for skip-row
+ * stack levels that do not fit in shared memory.  Some callers cannot allow
+ * that: cudaMalloc can wait until the whole device is idle, which a serving
+ * loop with a latency budget cannot afford, and a process whose device memory
+ * is already handed out by its own caching allocator may not get a raw
+ * allocation at all.  This variant keeps those levels in a fixed 16 MiB array
+ * of the library's device memory (every GPU that loads the library holds it
+ * until the process exits) and calls no allocating routine.
+ * Arguments, results and bit layout are exactly those of pp_tree_dp, and
+ * pp_traceback reads the bits as usual.
+ * Limit: batch * (stack levels beyond shared memory) * padded columns * 8
+ * bytes must be at most 16 MiB (pp_dp_geometry gives the levels held in
+ * shared memory and the padded columns, pp_instance_preorder the stack
+ * depth); a larger launch is rejected with PP_EINVAL and nothing runs.
+ * The instance's device must be the current device.  The first call on a
+ * device looks up the array's device address (a one-time set-up); make that
+ * first call before any stream capture.  All calls on a device share the
+ * array and leave their contents in it.  Nothing in it needs to start at
+ * zero, since a call writes every stack level before reading it.  But calls
+ * that overlap on the GPU (other streams, other host threads) race on it and
+ * give wrong results: keep them ordered.
+ */
+pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const int64_t *profit,
+                             const int32_t *budget, int32_t max_budget, int64_t *best,
+                             uint32_t *bits, void *stream);
+
+/*
  * pp_traceback -- recover each item's optimal parent-closed set from the
  * decision bits (Algorithm 1, "backtrack from D[1,k]"): start at position 0
  * with j = k; "take" marks the chunk, j -= w_i and moves to i+1; "skip" moves

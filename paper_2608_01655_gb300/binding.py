@@ -61,6 +61,7 @@ _SIGS = {
     "pp_test_inject": [_i32, _i32],
     "pp_dp_geometry": [_P, _i32, _i32, _P],
     "pp_tune_dp": [_i32, _i32, _i32],
+    "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -193,6 +194,12 @@ def pp_dp_bits_size(inst: Instance, batch: int, max_budget: int) -> int:
 def pp_tree_dp(inst: Instance, profit, budget, max_budget: int, best, bits, stream=None):
     _check(_lib.pp_tree_dp(inst.handle, int(budget.shape[0]), _dev(profit), _dev(budget),
                            int(max_budget), _dev(best), _dev(bits), _stream(stream)))
+
+
+def pp_tree_dp_noalloc(inst: Instance, profit, budget, max_budget: int, best, bits, stream=None):
+    """pp_tree_dp without device allocation (fixed 16 MiB stack scratch per device)."""
+    _check(_lib.pp_tree_dp_noalloc(inst.handle, int(budget.shape[0]), _dev(profit), _dev(budget),
+                                   int(max_budget), _dev(best), _dev(bits), _stream(stream)))
 
 
 def pp_traceback(inst: Instance, bits, budget, max_budget: int, chosen, stream=None):

@@ -34,6 +34,7 @@
 // `lane` is column (g * 32 + lane) * C + c + 1.
 #include <algorithm>
 #include <climits>
+#include <mutex>
 
 #include "pp_internal.cuh"
 
@@ -798,21 +799,14 @@ static pp_status launch_flat_c(pp_instance *inst, int batch, const int64_t *prof
     return PP_OK;
 }
 
-pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
-                         const int32_t *item_budget, const int32_t *item_active, const DpGeom &g,
-                         int64_t *best, uint32_t *bits, cudaStream_t st, int32_t max_budget)
+// Launch the DP kernel selected by the geometry with the skip-row stack levels
+// below L_smem kept in `gstack` (batch * L_glob * kpad int64, may be null when
+// L_glob == 0).
+static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
+                                   const int32_t *item_budget, const int32_t *item_active,
+                                   const DpGeom &g, int64_t *best, uint32_t *bits, cudaStream_t st,
+                                   int32_t max_budget, int64_t *gstack, int L_glob)
 {
-    if (batch <= 0) return PP_OK;
-    if (inst->n == 0) {
-        PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
-        return PP_OK;
-    }
-    const int L_glob = inst->stack_depth - g.L_smem;
-    if (L_glob > 0) {
-        pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
-        if (s != PP_OK) return s;
-    }
-    int64_t *gstack = reinterpret_cast<int64_t *>(inst->stack.ptr);
     if (g.wave) {
         const void *fn = wave_kernel_for(g.C, g.WMAX);
         if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
@@ -849,6 +843,24 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
     case 32: return launch_flat_c<32>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
     default: return fail(PP_EINVAL, "unsupported DP geometry");
     }
+}
+
+pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
+                         const int32_t *item_budget, const int32_t *item_active, const DpGeom &g,
+                         int64_t *best, uint32_t *bits, cudaStream_t st, int32_t max_budget)
+{
+    if (batch <= 0) return PP_OK;
+    if (inst->n == 0) {
+        PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
+        return PP_OK;
+    }
+    const int L_glob = inst->stack_depth - g.L_smem;
+    if (L_glob > 0) {
+        pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
+        if (s != PP_OK) return s;
+    }
+    return launch_dp_kernels(inst, batch, profit, by_node, item_budget, item_active, g, best, bits, st,
+                             max_budget, reinterpret_cast<int64_t *>(inst->stack.ptr), L_glob);
 }
 
 pp_status launch_traceback(pp_instance *inst, int batch, const uint32_t *bits, const DpGeom &g,
@@ -936,4 +948,69 @@ extern "C" pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int3
     out[6] = (int32_t)g.smem;
     out[7] = g.kpad;
     return PP_OK;
+}
+
+// ===========================================================================
+// pp_tree_dp_noalloc: the same DP launch with the skip-row stack levels that do
+// not fit in shared memory kept in a fixed array of this library's device
+// memory instead of instance scratch, so the call never allocates.
+// ===========================================================================
+namespace pp {
+
+constexpr size_t kStaticStackBytes = (size_t)16 << 20;   // per device, held until the process exits
+static __device__ __align__(256) int64_t g_static_stack[kStaticStackBytes / sizeof(int64_t)];
+
+constexpr int kMaxDevices = 64;
+static std::mutex g_static_stack_mu;
+static int64_t *g_static_stack_addr[kMaxDevices] = {};
+
+// Device address of g_static_stack on `device`, resolved on first use with
+// that device current (host code cannot use the symbol itself as a pointer).
+static pp_status static_stack_address(int device, int64_t **out)
+{
+    if (device < 0 || device >= kMaxDevices) return fail(PP_EINVAL, "device ordinal out of range");
+    std::lock_guard<std::mutex> lock(g_static_stack_mu);
+    if (!g_static_stack_addr[device]) {
+        void *ptr = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&ptr, g_static_stack);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(fixed DP stack scratch)");
+        g_static_stack_addr[device] = reinterpret_cast<int64_t *>(ptr);
+    }
+    *out = g_static_stack_addr[device];
+    return PP_OK;
+}
+
+}  // namespace pp
+
+extern "C" pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const int64_t *profit,
+                                        const int32_t *budget, int32_t max_budget, int64_t *best,
+                                        uint32_t *bits, void *stream)
+{
+    if (!inst) return fail(PP_EINVAL, "null instance");
+    if (batch < 0) return fail(PP_EINVAL, "batch must be >= 0");
+    int cur_dev = -1;
+    PP_CUDA(cudaGetDevice(&cur_dev));
+    if (cur_dev != inst->device) return fail(PP_EINVAL, "the instance's device must be the current device");
+    int64_t *scratch = nullptr;
+    pp_status s = static_stack_address(cur_dev, &scratch);     // one-time set-up per device
+    if (s != PP_OK) return s;
+    DpGeom g;
+    if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
+    if (batch == 0) return PP_OK;
+    if (!budget || !best || (inst->n > 0 && (!profit || !bits)))
+        return fail(PP_EINVAL, "null device pointer");
+    cudaStream_t st = (cudaStream_t)stream;
+    if (inst->n == 0) {
+        PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
+        return PP_OK;
+    }
+    const int L_glob = inst->stack_depth - g.L_smem;
+    const size_t need = (size_t)batch * (size_t)std::max(L_glob, 0) * (size_t)g.kpad * sizeof(int64_t);
+    if (need > kStaticStackBytes)
+        return fail(PP_EINVAL, "pp_tree_dp_noalloc: this launch needs " + std::to_string(need) +
+                                   " bytes of skip-row stack scratch, more than its fixed " +
+                                   std::to_string(kStaticStackBytes) +
+                                   " bytes; use a smaller batch or pp_tree_dp");
+    return launch_dp_kernels(inst, batch, profit, true, budget, nullptr, g, best, bits, st, max_budget,
+                             scratch, L_glob);
 }
