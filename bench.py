@@ -365,6 +365,30 @@ def run_native(args):
     return 0
 
 
+def run_profile_dp(args):
+    """A small case for ncu: marginals then the tree DP of `--profile-dp B`
+    items of the paper-scale workload, launched twice (ncu captures the second)."""
+    import torch
+    torch.cuda.set_device(0)
+    from paper_2608_01655_gb300 import binding as pp
+    from paper_2608_01655_gb300 import workloads as wl
+    inst = wl.make(BENCH_CONFIG)
+    ppi = pp.Instance.from_workload(inst)
+    B, n, k = args.profile_dp, inst.n, int(inst.budget.max())
+    workers = torch.arange(B, dtype=torch.int32, device="cuda") % inst.W
+    masks = torch.zeros((B, n), dtype=torch.int32, device="cuda")
+    prof = torch.zeros((B, n), dtype=torch.int64, device="cuda")
+    bud = torch.full((B,), k, dtype=torch.int32, device="cuda")
+    best = torch.zeros(B, dtype=torch.int64, device="cuda")
+    bits = torch.zeros(pp.pp_dp_bits_size(ppi, B, k) // 4, dtype=torch.int32, device="cuda")
+    for _ in range(2):
+        pp.pp_marginals(ppi, workers, masks, prof)
+        pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
+    ppi.sync()
+    print(json.dumps({"profile_dp": B, "geometry": pp.pp_dp_geometry(ppi, B, k), "best": best.tolist()}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -373,7 +397,11 @@ def main():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--probe-iters", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-dp", type=int, default=0, metavar="B",
+                    help="only launch the tree DP of B items twice (a small case for ncu) and exit")
     args = ap.parse_args()
+    if args.profile_dp:
+        return run_profile_dp(args)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
