@@ -66,9 +66,11 @@ typedef struct {
     int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded) */
     int64_t dp_cells;              /* out: sum over executed DPs of n * k_h (Eq. 9 cells) */
     int32_t kernel_launches;       /* out: kernels launched by this call */
+    int64_t dp_rows_swept;         /* out: rows the DPs actually swept (pruned sweep), summed */
     int32_t time_phases;           /* in: nonzero = time the phases below with CUDA events */
     float phase_ms[3];             /* out (if time_phases): device time of the marginal,
-                                      tree-DP and traceback launches, summed over the plan */
+                                      tree-DP (with its row pruning) and traceback launches,
+                                      summed over the plan */
 } pp_plan_stats;
 
 /*
@@ -168,9 +170,12 @@ pp_status pp_marginals(pp_instance *inst, int32_t batch, const int32_t *worker,
                        const uint32_t *holder_mask, int64_t *profit, void *stream);
 
 /*
- * pp_dp_bits_size -- bytes of the decision-bit workspace that pp_tree_dp
- * writes and pp_traceback reads for `batch` items whose budgets are at most
- * `max_budget`.  Returns 0 for batch <= 0 or an invalid max_budget.
+ * pp_dp_bits_size -- bytes of the workspace that pp_tree_dp writes and
+ * pp_traceback reads for `batch` items whose budgets are at most
+ * `max_budget`: the decision bits plus the rows of the pruned sweep (rows
+ * strictly below a chunk whose strict descendants all have profit <= 0 never
+ * change a kept row's value or decision, so the DP skips them).  Returns 0 for
+ * batch <= 0 or an invalid max_budget.
  */
 size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_t max_budget);
 
@@ -293,11 +298,14 @@ pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_bud
 /*
  * pp_tune_dp -- process-wide override of the DP launch shape, for tuning
  * sweeps: CTAs per cluster (1..8, 0 = automatic), columns per thread (power
- * of two up to 16, 0 = automatic), force_flat != 0 selects the one-CTA kernel.
- * Later pp_dp_bits_size / pp_tree_dp / pp_traceback / pp_plan_run calls use
- * it, so set it before sizing workspaces.  Errors: PP_EINVAL.
+ * of two up to 16, 0 = automatic), force_flat != 0 selects the one-CTA kernel,
+ * no_prune != 0 sweeps every row instead of the pruned sweep (results are the
+ * same either way).  Later pp_dp_bits_size / pp_tree_dp / pp_traceback /
+ * pp_plan_run calls use it, so set it before sizing workspaces.
+ * Errors: PP_EINVAL.
  */
-pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat);
+pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
+                     int32_t no_prune);
 
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);

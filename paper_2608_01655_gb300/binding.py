@@ -43,7 +43,8 @@ class PPError(RuntimeError):
 class PlanStats(ctypes.Structure):
     _fields_ = [("per_start_objective", _P), ("per_start_sweeps", _P), ("per_start_accepted", _P),
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
-                ("kernel_launches", _i32), ("time_phases", _i32), ("phase_ms", ctypes.c_float * 3)]
+                ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
+                ("phase_ms", ctypes.c_float * 3)]
 
 
 _SIGS = {
@@ -60,7 +61,7 @@ _SIGS = {
     "pp_plan_run": [_P, _i32, _P, _i32, _P, _P, ctypes.POINTER(PlanStats), _P],
     "pp_test_inject": [_i32, _i32],
     "pp_dp_geometry": [_P, _i32, _i32, _P],
-    "pp_tune_dp": [_i32, _i32, _i32],
+    "pp_tune_dp": [_i32, _i32, _i32, _i32],
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
@@ -225,6 +226,7 @@ class PlanResult:
     dp_cells: int
     kernel_launches: int
     phase_ms: tuple = ()
+    dp_rows_swept: int = 0
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
@@ -236,7 +238,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     sw = np.zeros(S, np.int32)
     acc = np.zeros(S, np.int32)
     used = np.zeros((S, W), np.int32)
-    st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0,
+    st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0, 0,
                    int(bool(time_phases)))
     op = None
     if orders is not None:
@@ -248,7 +250,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                             ctypes.byref(st), _stream(stream)))
     return PlanResult(placement[:, :n].copy(), int(obj.value), int(st.best_start), per, sw, acc, used,
                       int(st.dp_count), int(st.dp_cells), int(st.kernel_launches),
-                      tuple(float(x) for x in st.phase_ms) if time_phases else ())
+                      tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept))
 
 
 def pp_test_inject(kind: int, value: int):
@@ -265,5 +267,7 @@ def pp_dp_geometry(inst: Instance, batch: int, max_budget: int) -> dict:
     return {k: int(v) for k, v in zip(keys, out)}
 
 
-def pp_tune_dp(cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: bool = False):
-    _check(_lib.pp_tune_dp(int(cluster_ctas), int(columns_per_thread), int(bool(force_flat))))
+def pp_tune_dp(cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: bool = False,
+               no_prune: bool = False):
+    _check(_lib.pp_tune_dp(int(cluster_ctas), int(columns_per_thread), int(bool(force_flat)),
+                           int(bool(no_prune))))

@@ -220,7 +220,8 @@ constexpr uint64_t kLapBit = 1ull << 63;
 
 template <int C, int WMAX>
 __global__ void __launch_bounds__(512, 1)
-k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ profit,
+k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
+               const int32_t *__restrict__ nkept, const int64_t *__restrict__ profit,
                const int32_t *__restrict__ order, const int32_t *__restrict__ wmeta,
                const int32_t *__restrict__ item_budget, int32_t max_budget,
                const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
@@ -279,6 +280,10 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ profit,
     const int64_t *Pp = profit + (size_t)item * n;
     uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
+    // the rows this item sweeps: all of them, or the kept rows of the pruned sweep
+    const int nrows = rowlist ? nkept[item] : n;
+    const int32_t *rows = rowlist ? rowlist + (size_t)item * n : nullptr;
+    const int nblk_item = (nrows + 31) / 32;
 
     int64_t cur[C], top[C];
 #pragma unroll
@@ -289,10 +294,10 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ profit,
     // row metadata, 32 rows per block: lane l loads row blk*32 + l one block
     // ahead and stages (p, m) in shared memory for the warp; rows past the
     // last one are no-ops (p = -inf, skip = the row just computed), so every
-    // warp sweeps nblk * 32 rows
+    // warp sweeps nblk_item * 32 rows
     auto load_meta = [&](int r, int64_t &pv, int32_t &mv) {
-        if (r < n) {
-            const int i = n - 1 - r;
+        if (r < nrows) {
+            const int i = rows ? rows[r] : n - 1 - r;
             pv = Pp[order ? order[i] : i];
             mv = wmeta[i];
         } else {
@@ -309,7 +314,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ profit,
 #pragma unroll
     for (int q = 0; q < WMAX; ++q) carry[q] = has_prev ? 0 : (q == WMAX - 1 ? 0 : kNeg);
 
-    for (int blk = 0; blk < nblk && !aborted; ++blk) {
+    for (int blk = 0; blk < nblk_item && !aborted; ++blk) {
         __syncwarp();
         my_meta[lane] = make_int4((int)(uint32_t)pnext, (int)(uint32_t)((uint64_t)pnext >> 32), mnext, 0);
         const uint32_t stack_rows = __ballot_sync(kFull, (mnext & kWaveStackOps) != 0);   // bit = row of the block
@@ -473,7 +478,8 @@ static size_t flat_smem_fixed(int kpad)
 
 template <int C>
 __global__ void __launch_bounds__(1024, 1)
-k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
+k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__restrict__ nkept,
+               const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
                const int32_t *__restrict__ wpre, const int32_t *__restrict__ meta,
                const int32_t *__restrict__ item_budget, int32_t max_budget,
                const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
@@ -508,6 +514,8 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
     const int64_t *Pp = profit + (size_t)item * n;
     const int nblk = (n + 31) / 32;
     uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)nblk * C * 32 + lane;
+    const int nrows = rowlist ? nkept[item] : n;
+    const int32_t *rows = rowlist ? rowlist + (size_t)item * n : nullptr;
     uint32_t wbits[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) wbits[c] = 0;
@@ -518,8 +526,8 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
         cur[c] = 0;
         srow[c * T + t] = 0;
     }
-    for (int x = t; x < kMetaRows && x < n; x += T) {
-        const int i = n - 1 - x;
+    for (int x = t; x < kMetaRows && x < nrows; x += T) {
+        const int i = rows ? rows[x] : n - 1 - x;
         sp[x] = Pp[order ? order[i] : i];
         sw[x] = wpre[i];
         sm[x] = meta[i];
@@ -528,12 +536,12 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
 
     int64_t nx_p = 0;
     int32_t nx_w = 0, nx_m = 0;
-    for (int r = 0; r < n; ++r) {
+    for (int r = 0; r < nrows; ++r) {
         const int blk = r / kMetaRows, off = r - blk * kMetaRows, buf = (blk & 1) * kMetaRows;
         if (off == 0) {
             const int x = (blk + 1) * kMetaRows + t;
-            if (t < kMetaRows && x < n) {
-                const int ii = n - 1 - x;
+            if (t < kMetaRows && x < nrows) {
+                const int ii = rows ? rows[x] : n - 1 - x;
                 nx_p = Pp[order ? order[ii] : ii];
                 nx_w = wpre[ii];
                 nx_m = meta[ii];
@@ -572,7 +580,7 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
             outr[c * T + t] = v;
             if (take) wbits[c] |= mrow;
         }
-        if ((r & 31) == 31 || r == n - 1) {
+        if ((r & 31) == 31 || r == nrows - 1) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
                 Bw[((size_t)(r >> 5) * C + c) * 32] = wbits[c];
@@ -589,7 +597,7 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
         if (off == kMetaRows - 1) {
             const int x = (blk + 1) * kMetaRows + t;
             const int nb = ((blk + 1) & 1) * kMetaRows;
-            if (t < kMetaRows && x < n) {
+            if (t < kMetaRows && x < nrows) {
                 sp[nb + t] = nx_p;
                 sw[nb + t] = nx_w;
                 sm[nb + t] = nx_m;
@@ -610,18 +618,25 @@ k_tree_dp_flat(int32_t n, const int64_t *__restrict__ profit, const int32_t *__r
 }
 
 // ===========================================================================
-// Traceback from (0, k): take -> mark b_i, j -= w_i, i += 1; skip -> i =
-// next(i); stop at i = n or j = 0.  One thread walks; the block first clears
-// the output.  Planner mode (acc.mask != nullptr): the update is accepted in
-// the greedy pass, or in refinement iff D[0][k] > sum of p_h over the current
-// T_h (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
+// Traceback from (0, k) (Algorithm 1, "backtrack"): at a visited row, take ->
+// mark b_i, j -= w_i and go to the next kept row; skip -> go to next(i); stop
+// at i = n or j = 0.  In kept-row order a take always moves from kept index t
+// to t - 1 (the next kept row in preorder, since a pruned interior is all
+// "skip"), and a skip moves to skip[t].  One warp walks and speculates each
+// round on two take-runs: lanes 0-15 on the run that starts at t, lanes 16-31
+// on the run that starts at u = skip[t] (used when row t itself is skipped);
+// with skip and skip2 tables every address of the round is known up front
+// (after the suffix weights for weighted trees).  A round resolves an optional
+// skip of t, one take-run and the skip that ends it.
+// Planner mode (acc.mask != nullptr): the update is accepted in the greedy
+// pass, or in refinement iff D[0][k] > sum of p_h over the current T_h
+// (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
 // replaces bit h of the holder masks by the traced set.
 // ===========================================================================
 __global__ void __launch_bounds__(256)
-k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int P, int kpad,
+k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
-            const int32_t *__restrict__ wpre, const int32_t *__restrict__ next,
-            uint8_t *__restrict__ chosen, AcceptArgs acc)
+            const int32_t *__restrict__ wpre, uint8_t *__restrict__ chosen, AcceptArgs acc)
 {
     const int item = blockIdx.x;
     uint32_t hbit = 0;
@@ -640,8 +655,9 @@ k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int P, int kpad
         for (int32_t x = threadIdx.x; x < n; x += blockDim.x) ch[x] = 0;
     }
     __syncthreads();
-    if (threadIdx.x != 0) return;
-    if (acc.mask && !acc.greedy) {
+    if (threadIdx.x >= 32) return;
+    const int lane = threadIdx.x;
+    if (acc.mask && !acc.greedy && lane == 0) {
         acc.improved[item] = 1;
         acc.accepted[item] += 1;
     }
@@ -649,22 +665,212 @@ k_traceback(int32_t n, const uint32_t *__restrict__ bits, int C, int P, int kpad
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
     const int nblk = (n + 31) / 32;
-    const uint32_t *Bi = bits + (size_t)item * P * (size_t)nblk * C * 32;
-    int32_t i = 0;
-    while (i < n && j > 0) {
-        const int q = j - 1;
+    const uint32_t *Bi = w.bits + (size_t)item * P * (size_t)nblk * C * 32;
+    const int32_t *rl = w.rowlist + (size_t)item * n;
+    const int32_t *sk = w.skip + (size_t)item * n, *sk2 = w.skip2 + (size_t)item * n;
+    const int32_t *ws = w.wsuf + (size_t)item * (n + 1);
+    const int nk = w.nkept[item];
+    auto bit = [&](int row, int col) -> uint32_t {           // decision of kept row `row`, column col >= 1
+        const int q = col - 1;
         const int tt = q / C, c = q - tt * C;
-        const int r = n - 1 - i;
-        const uint32_t word = Bi[(((size_t)(tt >> 5) * nblk + (r >> 5)) * C + c) * 32 + (tt & 31)];
-        if ((word >> (r & 31)) & 1u) {
-            if (M) M[i] |= hbit;
-            else chosen[(size_t)item * n + order[i]] = 1;
-            j -= wpre[i];
-            i += 1;
+        const uint32_t word = Bi[(((size_t)(tt >> 5) * nblk + (row >> 5)) * C + c) * 32 + (tt & 31)];
+        return (word >> (row & 31)) & 1u;
+    };
+    int t = nk - 1;                 // row of position 0 (the first root): swept last
+    int u = nk > 0 ? sk[t] : -1;
+    const int half = lane >> 4, l = lane & 15;
+    for (int guard = 0; guard <= n && t >= 0 && j > 0; ++guard) {
+        // lane (half, l): row `l` steps into the take-run from t (half 0) or u (half 1)
+        const int base = half ? u : t;
+        const int row = base - l;
+        const bool live = base >= 0 && row >= 0;
+        int col = j;
+        if (live && l > 0) col = unit_weights ? j - l : j - (ws[row + 1] - ws[base + 1]);
+        const bool take = live && col > 0 && bit(row, col);
+        const int pos = live ? rl[row] : -1;
+        const int s1 = live ? sk[row] : -1, s2 = live ? sk2[row] : -1;
+        const int wrow = live ? wpre[pos] : 0;
+        const uint32_t tm = __ballot_sync(kFull, take);
+        int h0;                                           // the half that continues the walk
+        if (tm & 1u) {
+            h0 = 0;
         } else {
-            i = next[i];
+            if (u < 0) break;                             // t skipped and next(t) = n: done
+            if (!(tm & 0x10000u)) {                       // u skipped too
+                const int nt = __shfl_sync(kFull, s1, 16), nu = __shfl_sync(kFull, s2, 16);
+                t = nt;
+                u = nu;
+                continue;
+            }
+            h0 = 1;
+        }
+        const uint32_t run = (tm >> (16 * h0)) & 0xFFFFu;
+        const int l0 = __ffs(~run) - 1 < 16 ? __ffs(~run) - 1 : 16;   // first lane of the half not taken
+        if (half == h0 && l < l0) {
+            if (M) M[pos] |= hbit;
+            else chosen[(size_t)item * n + order[pos]] = 1;
+        }
+        const int src = 16 * h0 + (l0 < 16 ? l0 : 15);
+        const int ecol = __shfl_sync(kFull, col, src);
+        const int erow = __shfl_sync(kFull, row, src);
+        const int es1 = __shfl_sync(kFull, s1, src), es2 = __shfl_sync(kFull, s2, src);
+        const int ew = __shfl_sync(kFull, wrow, src);
+        const int ebase = h0 ? u : t;
+        if (l0 == 16) {                                   // 16 takes: continue after the last
+            t = ebase - 16;
+            j = ecol - ew;
+            u = t >= 0 ? sk[t] : -1;
+            continue;
+        }
+        if (erow < 0 || ecol <= 0) break;                 // ran past position n-1 or out of slots
+        t = es1;                                          // row erow is skipped
+        u = es2;
+        j = ecol;
+    }
+}
+
+// ===========================================================================
+// Pruned sweep (one CTA per item).  A strict descendant set with no positive
+// profit is never worth taking: for a parent x whose strict descendants all
+// have p <= 0, D[x+1][.] = D[next(x)][.] (selecting nothing below x is
+// optimal), every decision bit below x is "skip", and the stack pushes and
+// pops of those rows balance.  So the rows strictly below x can be removed
+// from the sweep: row x then sees D[next(x)] as its row i+1, which is the same
+// values, and no kept row's value or bit changes.  With `cnt` the prefix
+// counts of positive profits in preorder, x has a positive strict descendant
+// iff cnt[next(x)] - cnt[x + 1] > 0, and row i is kept iff it is a root or its
+// parent has one.  Kept rows are listed in sweep order (decreasing i).
+// ===========================================================================
+__device__ __forceinline__ int block_exclusive_scan(int v, int *total, int *sh)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFull, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+        int w = lane < nw ? sh[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < nw) sh[lane] = w;           // inclusive warp totals
+    }
+    __syncthreads();
+    const int before = wid > 0 ? sh[wid - 1] : 0;
+    *total = sh[nw - 1];
+    __syncthreads();                           // sh is reused by the next scan
+    return before + x - v;
+}
+
+template <bool BYNODE>
+__global__ void __launch_bounds__(1024)
+k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
+        const int32_t *__restrict__ next, const int32_t *__restrict__ ppos,
+        const int32_t *__restrict__ wpre, const int32_t *__restrict__ item_active, DpWork w,
+        int prune, unsigned long long *__restrict__ rows_kept)
+{
+    __shared__ int sh[32];
+    const int item = blockIdx.x;
+    if (item_active && !item_active[item]) return;
+    const int64_t *Pp = profit + (size_t)item * n;
+    int32_t *cnt = w.cnt + (size_t)item * (n + 1);
+    int32_t *rl = w.rowlist + (size_t)item * n;
+    int32_t *kx = w.kidx + (size_t)item * n;
+    const int T = blockDim.x, t = threadIdx.x;
+    const int chunk = (n + T - 1) / T;
+    const int lo = min(n, t * chunk), hi = min(n, lo + chunk);
+    int total = 0;
+    // prefix counts of positive profits, preorder
+    int c = 0;
+    for (int i = lo; i < hi; ++i) c += Pp[BYNODE ? order[i] : i] > 0;
+    int ex = block_exclusive_scan(c, &total, sh);
+    for (int i = lo; i < hi; ++i) {
+        cnt[i] = ex;
+        ex += Pp[BYNODE ? order[i] : i] > 0;
+    }
+    if (t == 0) cnt[n] = total;
+    __syncthreads();
+    // kept rows in sweep order r = n - 1 - i
+    auto keep = [&](int i) -> bool {
+        if (!prune) return true;
+        const int pa = ppos[i];
+        return pa < 0 || cnt[next[pa]] - cnt[pa + 1] > 0;
+    };
+    int kc = 0;
+    for (int r = lo; r < hi; ++r) kc += keep(n - 1 - r);
+    int kex = block_exclusive_scan(kc, &total, sh);
+    for (int r = lo; r < hi; ++r) {
+        const int i = n - 1 - r;
+        if (keep(i)) {
+            rl[kex] = i;
+            kx[i] = kex++;
+        } else {
+            kx[i] = -1;
         }
     }
+    const int nk = total;
+    if (t == 0) {
+        w.nkept[item] = nk;
+        if (rows_kept) atomicAdd(rows_kept, (unsigned long long)nk);
+    }
+    __syncthreads();
+    // traceback tables over kept rows: skip targets and suffix weights
+    int32_t *sk = w.skip + (size_t)item * n, *sk2 = w.skip2 + (size_t)item * n;
+    int32_t *ws = w.wsuf + (size_t)item * (n + 1);
+    const int kchunk = (nk + T - 1) / T;
+    const int klo = min(nk, t * kchunk), khi = min(nk, klo + kchunk);
+    int wsum = 0;
+    for (int q = klo; q < khi; ++q) {
+        const int i = rl[q];
+        sk[q] = next[i] < n ? kx[next[i]] : -1;
+        wsum += wpre[i];
+    }
+    int wex = block_exclusive_scan(wsum, &total, sh);     // weight of kept rows before klo
+    for (int q = klo; q < khi; ++q) {
+        ws[q] = total - wex;                               // weight of kept rows q..nk-1
+        wex += wpre[rl[q]];
+    }
+    if (t == 0) ws[nk] = 0;
+    __syncthreads();
+    for (int q = klo; q < khi; ++q) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t dp_work_bytes(int batch, int n, int words)
+{
+    const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
+    return align256(B * nb * words * 4) + 4 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
+           align256(B * 4);
+}
+
+DpWork dp_work_split(void *base, int batch, int n, int words)
+{
+    const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
+    char *p = reinterpret_cast<char *>(base);
+    DpWork w;
+    w.bits = reinterpret_cast<uint32_t *>(p);
+    p += align256(B * nb * words * 4);
+    w.rowlist = reinterpret_cast<int32_t *>(p);
+    p += align256(B * N * 4);
+    w.kidx = reinterpret_cast<int32_t *>(p);
+    p += align256(B * N * 4);
+    w.cnt = reinterpret_cast<int32_t *>(p);
+    p += align256(B * (N + 1) * 4);
+    w.nkept = reinterpret_cast<int32_t *>(p);
+    p += align256(B * 4);
+    w.skip = reinterpret_cast<int32_t *>(p);
+    p += align256(B * N * 4);
+    w.skip2 = reinterpret_cast<int32_t *>(p);
+    p += align256(B * N * 4);
+    w.wsuf = reinterpret_cast<int32_t *>(p);
+    return w;
 }
 
 // ===========================================================================
@@ -691,7 +897,7 @@ static int max_smem_optin(const pp_instance *inst)
 }
 
 // Geometry overrides set by pp_tune_dp (0 = automatic).
-static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0;
+static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0, g_tune_noprune = 0;
 
 static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom *g)
 {
@@ -788,10 +994,12 @@ template <int C>
 static pp_status launch_flat_c(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
                                const int32_t *item_budget, int32_t max_budget,
                                const int32_t *item_active, const DpGeom &g, int64_t *best,
-                               uint32_t *bits, int64_t *gstack, int L_glob, cudaStream_t st)
+                               const DpWork &work, int64_t *gstack, int L_glob, cudaStream_t st)
 {
+    uint32_t *bits = work.bits;
     PP_CUDA(cudaFuncSetAttribute(k_tree_dp_flat<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem));
-    k_tree_dp_flat<C><<<batch, g.T, g.smem, st>>>(inst->n, profit, by_node ? inst->d_order : nullptr,
+    k_tree_dp_flat<C><<<batch, g.T, g.smem, st>>>(inst->n, work.rowlist, work.nkept, profit,
+                                                   by_node ? inst->d_order : nullptr,
                                                    inst->d_wpre, inst->d_meta, item_budget, max_budget,
                                                    item_active, best, bits, gstack, g.L_smem, L_glob,
                                                    inst->d_status);
@@ -804,9 +1012,20 @@ static pp_status launch_flat_c(pp_instance *inst, int batch, const int64_t *prof
 // L_glob == 0).
 static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
                                    const int32_t *item_budget, const int32_t *item_active,
-                                   const DpGeom &g, int64_t *best, uint32_t *bits, cudaStream_t st,
-                                   int32_t max_budget, int64_t *gstack, int L_glob)
+                                   const DpGeom &g, int64_t *best, const DpWork &work, cudaStream_t st,
+                                   int32_t max_budget, int64_t *gstack, int L_glob,
+                                   unsigned long long *rows_kept)
 {
+    // the pruned sweep of every item, then the DP over its kept rows
+    if (by_node)
+        k_prune<true><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_ppos,
+                                              inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
+    else
+        k_prune<false><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_ppos,
+                                               inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
+    PP_CUDA(cudaGetLastError());
+    uint32_t *bits = work.bits;
+    const int32_t *rowlist = work.rowlist, *nkept = work.nkept;
     if (g.wave) {
         const void *fn = wave_kernel_for(g.C, g.WMAX);
         if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
@@ -829,25 +1048,26 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
         const int32_t *wm = inst->d_wave;
         int32_t L_smem = g.L_smem, Lg = L_glob;
         int32_t *status = inst->d_status;
-        void *args[] = {&n, &nblk, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
+        void *args[] = {&n, &nblk, (void *)&rowlist, (void *)&nkept, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
                         (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status};
         PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
         return PP_OK;
     }
     switch (g.C) {
-    case 1: return launch_flat_c<1>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
-    case 2: return launch_flat_c<2>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
-    case 4: return launch_flat_c<4>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
-    case 8: return launch_flat_c<8>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
-    case 16: return launch_flat_c<16>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
-    case 32: return launch_flat_c<32>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, bits, gstack, L_glob, st);
+    case 1: return launch_flat_c<1>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
+    case 2: return launch_flat_c<2>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
+    case 4: return launch_flat_c<4>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
+    case 8: return launch_flat_c<8>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
+    case 16: return launch_flat_c<16>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
+    case 32: return launch_flat_c<32>(inst, batch, profit, by_node, item_budget, max_budget, item_active, g, best, work, gstack, L_glob, st);
     default: return fail(PP_EINVAL, "unsupported DP geometry");
     }
 }
 
 pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
                          const int32_t *item_budget, const int32_t *item_active, const DpGeom &g,
-                         int64_t *best, uint32_t *bits, cudaStream_t st, int32_t max_budget)
+                         int64_t *best, const DpWork &work, cudaStream_t st, int32_t max_budget,
+                         unsigned long long *rows_kept)
 {
     if (batch <= 0) return PP_OK;
     if (inst->n == 0) {
@@ -859,19 +1079,19 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
         pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
         if (s != PP_OK) return s;
     }
-    return launch_dp_kernels(inst, batch, profit, by_node, item_budget, item_active, g, best, bits, st,
-                             max_budget, reinterpret_cast<int64_t *>(inst->stack.ptr), L_glob);
+    return launch_dp_kernels(inst, batch, profit, by_node, item_budget, item_active, g, best, work, st,
+                             max_budget, reinterpret_cast<int64_t *>(inst->stack.ptr), L_glob, rows_kept);
 }
 
-pp_status launch_traceback(pp_instance *inst, int batch, const uint32_t *bits, const DpGeom &g,
+pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, const DpGeom &g,
                            const int32_t *item_budget, uint8_t *chosen, const AcceptArgs *acc,
                            cudaStream_t st)
 {
     if (batch <= 0 || inst->n == 0) return PP_OK;
     AcceptArgs a;
     if (acc) a = *acc;
-    k_traceback<<<batch, 256, 0, st>>>(inst->n, bits, g.C, g.P, g.kpad, item_budget, inst->d_order,
-                                       inst->d_wpre, inst->d_next, chosen, a);
+    k_traceback<<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
+                                       inst->d_order, inst->d_wpre, chosen, a);
     PP_CUDA(cudaGetLastError());
     return PP_OK;
 }
@@ -884,7 +1104,7 @@ extern "C" size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_
 {
     DpGeom g;
     if (!inst || batch <= 0 || !dp_geometry(inst, max_budget, &g, batch)) return 0;
-    return (size_t)batch * (size_t)((inst->n + 31) / 32 * 32) * (size_t)g.words * sizeof(uint32_t);
+    return dp_work_bytes(batch, inst->n, g.words);
 }
 
 extern "C" pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t *profit,
@@ -898,8 +1118,8 @@ extern "C" pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t 
     if (batch == 0) return PP_OK;
     if (!budget || !best || (inst->n > 0 && (!profit || !bits)))
         return fail(PP_EINVAL, "null device pointer");
-    return launch_tree_dp(inst, batch, profit, true, budget, nullptr, g, best, bits,
-                          (cudaStream_t)stream, max_budget);
+    return launch_tree_dp(inst, batch, profit, true, budget, nullptr, g, best,
+                          dp_work_split(bits, batch, inst->n, g.words), (cudaStream_t)stream, max_budget);
 }
 
 extern "C" pp_status pp_traceback(pp_instance *inst, int32_t batch, const uint32_t *bits,
@@ -912,7 +1132,8 @@ extern "C" pp_status pp_traceback(pp_instance *inst, int32_t batch, const uint32
     if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
     if (batch == 0 || inst->n == 0) return PP_OK;
     if (!bits || !budget || !chosen) return fail(PP_EINVAL, "null device pointer");
-    return launch_traceback(inst, batch, bits, g, budget, chosen, nullptr, (cudaStream_t)stream);
+    return launch_traceback(inst, batch, dp_work_split(const_cast<uint32_t *>(bits), batch, inst->n, g.words), g,
+                            budget, chosen, nullptr, (cudaStream_t)stream);
 }
 
 extern "C" pp_status pp_test_inject(int32_t kind, int32_t value)
@@ -922,7 +1143,8 @@ extern "C" pp_status pp_test_inject(int32_t kind, int32_t value)
     return PP_OK;
 }
 
-extern "C" pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat)
+extern "C" pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
+                                int32_t no_prune)
 {
     if (cluster_ctas < 0 || cluster_ctas > 8 || columns_per_thread < 0 || columns_per_thread > 16 ||
         (columns_per_thread & (columns_per_thread - 1)) != 0)
@@ -930,6 +1152,7 @@ extern "C" pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread
     g_tune_cl = cluster_ctas;
     g_tune_c = columns_per_thread;
     g_tune_flat = force_flat != 0;
+    g_tune_noprune = no_prune != 0;
     return PP_OK;
 }
 
@@ -1011,6 +1234,7 @@ extern "C" pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const 
                                    " bytes of skip-row stack scratch, more than its fixed " +
                                    std::to_string(kStaticStackBytes) +
                                    " bytes; use a smaller batch or pp_tree_dp");
-    return launch_dp_kernels(inst, batch, profit, true, budget, nullptr, g, best, bits, st, max_budget,
-                             scratch, L_glob);
+    return launch_dp_kernels(inst, batch, profit, true, budget, nullptr, g, best,
+                             dp_work_split(bits, batch, inst->n, g.words), st, max_budget, scratch, L_glob,
+                             nullptr);
 }

@@ -215,6 +215,7 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     cudaFree(inst->d_wpre);
     cudaFree(inst->d_meta);
     cudaFree(inst->d_wave);
+    cudaFree(inst->d_ppos);
     cudaFree(inst->d_budget);
     cudaFree(inst->d_a);
     cudaFree(inst->d_delta);
@@ -291,6 +292,16 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if ((s = upload(&inst->d_wpre, inst->h_wpre.data(), n, st))) return s;
     if ((s = upload(&inst->d_meta, inst->h_meta.data(), n, st))) return s;
     if ((s = upload(&inst->d_wave, inst->h_wave.data(), n, st))) return s;
+    {
+        std::vector<int32_t> pos(n), ppos(n);
+        for (int32_t i = 0; i < n; ++i) pos[inst->h_order[i]] = i;
+        for (int32_t i = 0; i < n; ++i) {
+            const int32_t par = parent[inst->h_order[i]];
+            ppos[i] = par < 0 ? -1 : pos[par];
+        }
+        if ((s = upload(&inst->d_ppos, ppos.data(), n, st))) return s;
+        PP_CUDA(cudaStreamSynchronize(st));          // the host vectors die here
+    }
     if ((s = upload(&inst->d_budget, budget, W, st))) return s;
     PP_CUDA(cudaMalloc(&inst->d_status, sizeof(int32_t)));
     PP_CUDA(cudaMemsetAsync(inst->d_status, 0, sizeof(int32_t), st));

@@ -74,6 +74,29 @@ struct DpGeom {
 // holds the take decisions of column (g * 32 + lane) * C + c + 1, with
 // nblk = ceil(n / 32).
 
+// Workspace of one batched DP launch (pp_dp_bits_size bytes, carved in this
+// order): decision bits, then the pruned sweep (rows kept in sweep order, the
+// inverse map position -> kept index or -1, prefix counts of positive
+// profits, kept-row counts).  A row is dropped when every strict descendant
+// of its parent has a non-positive profit: such a parent's interior is never
+// taken and leaves D[parent+1] = D[next(parent)], so dropping those rows
+// changes no value and no bit of a kept row (see k_prune).
+// For the traceback, per kept row t (kept index, sweep order): skip[t] = kept
+// index of next(row t), -1 when next(row t) = n; skip2[t] = skip[skip[t]]
+// (-1 propagates); wsuf[t] = sum of the weights of kept rows t..nkept-1.
+struct DpWork {
+    uint32_t *bits = nullptr;      // [batch][P][nblk][C][32]
+    int32_t *rowlist = nullptr;    // [batch][n]
+    int32_t *kidx = nullptr;       // [batch][n]
+    int32_t *cnt = nullptr;        // [batch][n + 1]
+    int32_t *nkept = nullptr;      // [batch]
+    int32_t *skip = nullptr;       // [batch][n]
+    int32_t *skip2 = nullptr;      // [batch][n]
+    int32_t *wsuf = nullptr;       // [batch][n + 1]
+};
+size_t dp_work_bytes(int batch, int n, int words);
+DpWork dp_work_split(void *base, int batch, int n, int words);
+
 // Status word values written by kernels (same numbering as pp_status).
 constexpr int32_t kDevOk = PP_OK;
 
@@ -100,6 +123,7 @@ struct pp_instance {
     int32_t *d_wpre = nullptr;          // [n] chunk weight
     int32_t *d_meta = nullptr;          // [n] packed skip / push codes
     int32_t *d_wave = nullptr;          // [n] wavefront-kernel row metadata
+    int32_t *d_ppos = nullptr;          // [n] preorder position of the parent, -1 for roots
     int32_t *d_budget = nullptr;        // [W]
     int64_t *d_a = nullptr;             // mode 0: [W][n] a_m(b)       (Eq. 2)
     int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)
@@ -133,8 +157,8 @@ bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int bat
 //   item_budget:  [batch] budgets; item_active: [batch] or null (0 = skip item)
 pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool prof_by_node,
                          const int32_t *item_budget, const int32_t *item_active,
-                         const DpGeom &g, int64_t *best, uint32_t *bits, cudaStream_t st,
-                         int32_t max_budget);
+                         const DpGeom &g, int64_t *best, const DpWork &work, cudaStream_t st,
+                         int32_t max_budget, unsigned long long *rows_kept = nullptr);
 
 pp_status launch_marginals(pp_instance *inst, int batch, const int32_t *worker,
                            const uint32_t *mask, bool by_node, const int32_t *item_active,
@@ -156,7 +180,7 @@ struct AcceptArgs {
     uint32_t *mask = nullptr;           // [batch][n] holder masks (preorder)
     int greedy = 0;                     // 1: always accept (WorkerGreedy pass)
 };
-pp_status launch_traceback(pp_instance *inst, int batch, const uint32_t *bits, const DpGeom &g,
+pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, const DpGeom &g,
                            const int32_t *item_budget, uint8_t *chosen, const AcceptArgs *acc,
                            cudaStream_t st);
 

@@ -45,6 +45,7 @@ struct PlanBuffers {
     int32_t *sweeps;     // [B]
     int32_t *work;       // [W + 1][B]: step workers, then standalone ids
     int32_t *kbud;       // [W + 1][B]: step budgets, then standalone budgets
+    unsigned long long *rows;   // [1] DP rows swept (pruned sweep) over the plan
 };
 
 static size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -53,11 +54,11 @@ static pp_status plan_buffers(pp_instance *inst, int B, PlanBuffers *pb)
 {
     const size_t n = (size_t)std::max(inst->n, 1);
     const int W = inst->W;
-    size_t off[11], tot = 0;
-    const size_t sz[11] = {4 * n * B, 8 * n * B, 8 * (size_t)B, 8 * (size_t)B, 8 * (size_t)B,
+    size_t off[12], tot = 0;
+    const size_t sz[12] = {4 * n * B, 8 * n * B, 8 * (size_t)B, 8 * (size_t)B, 8 * (size_t)B,
                            4 * (size_t)B, 4 * (size_t)B, 4 * (size_t)B, 4 * (size_t)B,
-                           4 * (size_t)(W + 1) * B, 4 * (size_t)(W + 1) * B};
-    for (int x = 0; x < 11; ++x) {
+                           4 * (size_t)(W + 1) * B, 4 * (size_t)(W + 1) * B, 8};
+    for (int x = 0; x < 12; ++x) {
         off[x] = tot;
         tot += align_up(sz[x]);
     }
@@ -75,6 +76,7 @@ static pp_status plan_buffers(pp_instance *inst, int B, PlanBuffers *pb)
     pb->sweeps = reinterpret_cast<int32_t *>(base + off[8]);
     pb->work = reinterpret_cast<int32_t *>(base + off[9]);
     pb->kbud = reinterpret_cast<int32_t *>(base + off[10]);
+    pb->rows = reinterpret_cast<unsigned long long *>(base + off[11]);
     return PP_OK;
 }
 
@@ -99,10 +101,12 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
     PlanBuffers pb;
     pp_status s = plan_buffers(inst, B, &pb);
     if (s != PP_OK) return s;
-    const size_t nb = (size_t)std::max((n + 31) / 32 * 32, 32);
-    s = ensure_scratch(inst->plan_bits, std::max((size_t)S * g.words, (size_t)W * gw.words) * nb * sizeof(uint32_t));
+    s = ensure_scratch(inst->plan_bits, std::max(dp_work_bytes(S, n, g.words), dp_work_bytes(W, n, gw.words)));
     if (s != PP_OK) return s;
-    uint32_t *bits = reinterpret_cast<uint32_t *>(inst->plan_bits.ptr);
+    const DpWork work = dp_work_split(inst->plan_bits.ptr, S, n, g.words);
+    const DpWork work_w = dp_work_split(inst->plan_bits.ptr, W, n, gw.words);
+    unsigned long long *rows_kept = pb.rows;
+    PP_CUDA(cudaMemsetAsync(rows_kept, 0, sizeof(unsigned long long), st));
 
     // ---- start orders -----------------------------------------------------
     std::vector<int32_t> ord((size_t)S * W);
@@ -128,8 +132,10 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
             PP_CUDA(cudaMemcpyAsync(d_kb, kb.data(), 4 * W, cudaMemcpyHostToDevice, st));
             PP_CUDA(cudaMemsetAsync(pb.mask, 0, (size_t)4 * std::max(n, 1) * W, st));
             if ((s = launch_marginals(inst, W, d_ids, pb.mask, false, nullptr, pb.profit, nullptr, st))) return s;
-            if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, gw, pb.best, bits, st, maxk))) return s;
-            launches += 2;
+            if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, gw, pb.best, work_w, st, maxk,
+                                    rows_kept)))
+                return s;
+            launches += 3;
             std::vector<int64_t> score(W);
             standalone_cells = (int64_t)n * sumk;
             PP_CUDA(cudaMemcpyAsync(score.data(), pb.best, 8 * W, cudaMemcpyDeviceToHost, st));
@@ -187,7 +193,8 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         if ((r = mark())) return r;
         if ((r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st))) return r;
         if ((r = mark())) return r;
-        if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, bits, st, maxk))) return r;
+        if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, work, st, maxk, rows_kept)))
+            return r;
         if ((r = mark())) return r;
         AcceptArgs a;
         a.worker = wk;
@@ -198,9 +205,9 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         a.accepted = pb.accepted;
         a.mask = pb.mask;
         a.greedy = greedy;
-        if ((r = launch_traceback(inst, S, bits, g, kb, nullptr, &a, st))) return r;
+        if ((r = launch_traceback(inst, S, work, g, kb, nullptr, &a, st))) return r;
         if ((r = mark())) return r;
-        launches += 3;
+        launches += 4;
         return PP_OK;
     };
 
@@ -233,6 +240,8 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
     launches += 1;
     std::vector<int64_t> obj(S);
     std::vector<int32_t> sw(S), acc(S);
+    unsigned long long rows_swept = 0;
+    PP_CUDA(cudaMemcpyAsync(&rows_swept, rows_kept, sizeof(rows_swept), cudaMemcpyDeviceToHost, st));
     PP_CUDA(cudaMemcpyAsync(obj.data(), pb.obj, 8 * S, cudaMemcpyDeviceToHost, st));
     PP_CUDA(cudaMemcpyAsync(sw.data(), pb.sweeps, 4 * S, cudaMemcpyDeviceToHost, st));
     PP_CUDA(cudaMemcpyAsync(acc.data(), pb.accepted, 4 * S, cudaMemcpyDeviceToHost, st));
@@ -264,6 +273,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         stats->dp_count = dp_count;
         stats->dp_cells = cells;
         stats->kernel_launches = launches;
+        stats->dp_rows_swept = (int64_t)rows_swept;
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
         for (size_t x = 0; x + 3 < ev.size(); x += 4) {
             float a = 0.f, b = 0.f, c = 0.f;

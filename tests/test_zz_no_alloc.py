@@ -87,7 +87,7 @@ def test_noalloc_matches_tree_dp_twice(pp, w_max, tune):
             np.testing.assert_array_equal(got[2], ref[2])
         ppi.close()
     finally:
-        pp.pp_tune_dp(0, 0, False)
+        pp.pp_tune_dp(0, 0, False, False)
 
 
 def test_noalloc_rejects_oversized_launch(pp):
