@@ -270,10 +270,12 @@ def run_native(args):
     ppi.sync()
     dp_t = statistics.mean(dp_times)
     cells_launch = S * n * k
+    rows_swept = int(pp.pp_dp_rows_swept(ppi, S, k, bits).sum())
+    cells_swept = rows_swept * k
     peaks, peak_kind = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = SM_COUNT * 4 * 32 * sm_mhz * 1e6 / ALU_OPS_PER_CELL      # cells/s, issue-bound
-    achieved = cells_launch / dp_t
+    achieved = cells_swept / dp_t                 # cells the kernel actually computed
     # algorithmic bytes of one launch: decision bits + p/w/next + skip-row pushes
     order, nxt, skipc, pushl, depth = pp.pp_row_plan(inst.parent)
     pushes = int((pushl >= 0).sum())
@@ -286,7 +288,8 @@ def run_native(args):
                 "frac": achieved / alu_peak, "traffic": traffic,
                 "peak_source": f"derived: {SM_COUNT} SMs x 4 SMSP x 32 lanes x {sm_mhz:.0f} MHz / "
                                f"{ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
-                "kernel": "k_tree_dp", "launch_ms": 1000 * dp_t, "cells_per_launch": cells_launch,
+                "kernel": "k_tree_dp_wave", "launch_ms": 1000 * dp_t, "cells_per_launch": cells_launch,
+                "cells_swept_per_launch": cells_swept, "rows_swept_per_launch": rows_swept,
                 "hbm_bmin_gbs": bmin / dp_t / 1e9,
                 "hbm_bmin_frac": bmin / dp_t / 1e9 / float(peaks.get("hbm_gbs", 6800.0)),
                 "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0)), "hbm_peak_kind": peak_kind}
@@ -351,6 +354,7 @@ def run_native(args):
             "clocks": clocks,
             "plan": {"objective": best_obj, "best_rank": best_rank, "best_start": res.best_start,
                      "dp_count": res.dp_count, "dp_cells": cells_per_plan,
+                     "dp_rows_swept": phased.dp_rows_swept, "dp_cells_swept": phased.dp_rows_swept * k,
                      "sweeps": res.per_start_sweeps.tolist(),
                      "step_ms": [round(1000 * t, 3) for t in times]},
             "marginals_launch_ms": 1000 * statistics.mean(mg_times),

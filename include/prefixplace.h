@@ -230,6 +230,15 @@ pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const int64_t *pr
                              uint32_t *bits, void *stream);
 
 /*
+ * pp_dp_rows_swept -- for the last pp_tree_dp / pp_tree_dp_noalloc on
+ * `workspace` (same batch and max_budget), the number of rows each item's DP
+ * actually swept after pruning (host [batch] out).  Synchronises `stream`.
+ * Errors: PP_EINVAL, PP_ECUDA.
+ */
+pp_status pp_dp_rows_swept(const pp_instance *inst, int32_t batch, int32_t max_budget,
+                           const uint32_t *workspace, int32_t *rows, void *stream);
+
+/*
  * pp_traceback -- recover each item's optimal parent-closed set from the
  * decision bits (Algorithm 1, "backtrack from D[1,k]"): start at position 0
  * with j = k; "take" marks the chunk, j -= w_i and moves to i+1; "skip" moves

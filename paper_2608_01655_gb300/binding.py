@@ -63,6 +63,7 @@ _SIGS = {
     "pp_dp_geometry": [_P, _i32, _i32, _P],
     "pp_tune_dp": [_i32, _i32, _i32, _i32],
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
+    "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -201,6 +202,14 @@ def pp_tree_dp_noalloc(inst: Instance, profit, budget, max_budget: int, best, bi
     """pp_tree_dp without device allocation (fixed 16 MiB stack scratch per device)."""
     _check(_lib.pp_tree_dp_noalloc(inst.handle, int(budget.shape[0]), _dev(profit), _dev(budget),
                                    int(max_budget), _dev(best), _dev(bits), _stream(stream)))
+
+
+def pp_dp_rows_swept(inst: Instance, batch: int, max_budget: int, bits, stream=None) -> np.ndarray:
+    """Rows each item of the last DP on `bits` swept after pruning."""
+    rows = np.zeros(max(int(batch), 1), np.int32)
+    _check(_lib.pp_dp_rows_swept(inst.handle, int(batch), int(max_budget), _dev(bits), _host(rows),
+                                 _stream(stream)))
+    return rows[:int(batch)]
 
 
 def pp_traceback(inst: Instance, bits, budget, max_budget: int, chosen, stream=None):

@@ -170,7 +170,7 @@ __host__ __device__ inline size_t wave_fixed_bytes(int WPC, int WMAX)
 // own registers for c >= W, the left neighbour lane for c < W, and for lane 0
 // the boundary values bnd[q] = D[i+1][base - WMAX + 1 + q] of the previous warp.
 template <int C, int WMAX, int W>
-__device__ __forceinline__ void shift_by(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], int lane,
+__device__ __forceinline__ void shift_by(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], bool lane0,
                                          int64_t (&sh)[C])
 {
 #pragma unroll
@@ -179,13 +179,13 @@ __device__ __forceinline__ void shift_by(const int64_t (&cur)[C], const int64_t 
             sh[c] = cur[c - W];
         } else {
             const int64_t v = __shfl_up_sync(kFull, cur[C - W + c], 1);
-            sh[c] = lane == 0 ? bnd[WMAX - W + c] : v;
+            sh[c] = lane0 ? bnd[WMAX - W + c] : v;
         }
     }
 }
 
 template <int C, int WMAX>
-__device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], int lane,
+__device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], bool lane,
                                           int w, int64_t (&sh)[C])
 {
     if (WMAX == 1) {
@@ -276,10 +276,12 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
     uint32_t ack_seen = 0;
     bool aborted = false;
     const bool publish = has_next && lane == 31 && g != g_drop_publish_warp;   // this lane stores
+    const bool lane0 = lane == 0;
 
     const int64_t *Pp = profit + (size_t)item * n;
     uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
+    int64_t *const my_stk = stk + threadIdx.x, *const my_gst = gst + threadIdx.x;
     // the rows this item sweeps: all of them, or the kept rows of the pruned sweep
     const int nrows = rowlist ? nkept[item] : n;
     const int32_t *rows = rowlist ? rowlist + (size_t)item * n : nullptr;
@@ -316,7 +318,8 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
 
     for (int blk = 0; blk < nblk_item && !aborted; ++blk) {
         __syncwarp();
-        my_meta[lane] = make_int4((int)(uint32_t)pnext, (int)(uint32_t)((uint64_t)pnext >> 32), mnext, 0);
+        my_meta[lane] = make_int4((int)(uint32_t)pnext, (int)(uint32_t)((uint64_t)pnext >> 32), mnext,
+                                  (mnext & (3 << 3)) == (kWaveCur << 3));
         const uint32_t stack_rows = __ballot_sync(kFull, (mnext & kWaveStackOps) != 0);   // bit = row of the block
         __syncwarp();
         load_meta((blk + 1) * 32 + lane, pnext, mnext);
@@ -339,6 +342,8 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
             const uint64_t lap = (uint64_t)((r0 / kRing) & 1) << 63;
             const uint64_t *sl = my_ring + (size_t)(r0 & (kRing - 1)) * WMAX;
             uint64_t sv[WMAX == 1 ? kSub : 1];
+#pragma unroll
+            for (int u = 0; u < (WMAX == 1 ? kSub : 1); ++u) sv[u] = 0;
             if (has_prev) {
                 auto ready = [&] {
                     uint64_t bad = 0;
@@ -374,20 +379,25 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
                 const int64_t p = (int64_t)(((uint64_t)(uint32_t)mm.y << 32) | (uint32_t)mm.x);
                 const int32_t m = mm.z;
                 // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
+                // (the first warp's sv is all zero: column 0 of every row is 0)
                 int64_t bnd[WMAX];
-                if (u == 0 || !has_prev) {
+                if (u == 0) {
 #pragma unroll
                     for (int q = 0; q < WMAX; ++q) bnd[q] = carry[q];
                 } else if (WMAX == 1) {
                     bnd[0] = (int64_t)(sv[WMAX == 1 ? u - 1 : 0] & ~kLapBit);
-                } else {
+                } else if (has_prev) {
 #pragma unroll
                     for (int q = 0; q < WMAX; ++q) bnd[q] = (int64_t)(sl[(u - 1) * WMAX + q] & ~kLapBit);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < WMAX; ++q) bnd[q] = carry[q];
                 }
                 int64_t sh[C];
-                shift_row<C, WMAX>(cur, bnd, lane, (m & 7) + 1, sh);
-                const bool from_cur = (m & (3 << 3)) == (kWaveCur << 3);
+                shift_row<C, WMAX>(cur, bnd, lane0, (m & 7) + 1, sh);
                 const uint32_t mrow = mbase << u;
+                // skip row: row i+1 (a leaf) or the stack top
+                const bool from_cur = mm.w != 0;
 #pragma unroll
                 for (int c = 0; c < C; ++c) {
                     const int64_t sk = from_cur ? cur[c] : top[c];
@@ -404,20 +414,20 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
                         st_relaxed_cluster_u64_if(publish, sa + q * 8, (uint64_t)cur[C - WMAX + q] | lap);
                 }
                 // skip-row stack: push (the new row becomes the top), reload or reset the top
-                if (STACK && (m & kWaveStackOps)) {
+                // (the flags are the same in every lane; the vote makes that visible)
+                if (STACK && __any_sync(kFull, (m & kWaveStackOps) != 0)) {
                     const int lvl = (int)((uint32_t)m >> 16);
+                    int64_t *at = lvl < L_smem ? my_stk + (size_t)lvl * C * NT
+                                               : my_gst + (size_t)(lvl - L_smem) * CL * C * NT;
                     if (m & kWavePush) {
 #pragma unroll
                         for (int c = 0; c < C; ++c) {
                             top[c] = cur[c];
-                            if (lvl < L_smem) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
-                            else gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x] = cur[c];
+                            at[(size_t)c * NT] = cur[c];
                         }
                     } else if (m & kWaveReload) {
 #pragma unroll
-                        for (int c = 0; c < C; ++c)
-                            top[c] = lvl < L_smem ? stk[((size_t)lvl * C + c) * NT + threadIdx.x]
-                                                  : gst[((size_t)(lvl - L_smem) * CL * C + c) * NT + threadIdx.x];
+                        for (int c = 0; c < C; ++c) top[c] = at[(size_t)c * NT];
                     } else {
 #pragma unroll
                         for (int c = 0; c < C; ++c) top[c] = 0;
@@ -908,10 +918,13 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     const int64_t max_cl = std::max<int64_t>(1, (k + 32 * WMAX - 1) / (32 * WMAX));
     int cl_hi = (int)std::min<int64_t>(per_item, max_cl);
     if (g_tune_cl > 0) cl_hi = std::min(g_tune_cl, 8);
+    // Shape chosen by timing whole plans (paper-scale and source-dependent
+    // workloads): the widest cluster the SMs per item allow, then columns per
+    // thread grown until a CTA has at most 4 warps (one per scheduler).
     for (int CL = cl_hi; CL >= 1; --CL) {
         const int64_t cols = (k + CL - 1) / CL;
         int C = WMAX;
-        while ((cols + 32 * C - 1) / (32 * C) > 8 && C < 8) C *= 2;
+        while ((cols + 32 * C - 1) / (32 * C) > 4 && C < 8) C *= 2;
         if (g_tune_c > 0) C = std::max(std::min(g_tune_c, 8), WMAX);
         const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
         if (WPC > 16) continue;
@@ -1237,4 +1250,22 @@ extern "C" pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const 
     return launch_dp_kernels(inst, batch, profit, true, budget, nullptr, g, best,
                              dp_work_split(bits, batch, inst->n, g.words), st, max_budget, scratch, L_glob,
                              nullptr);
+}
+
+extern "C" pp_status pp_dp_rows_swept(const pp_instance *inst, int32_t batch, int32_t max_budget,
+                                      const uint32_t *workspace, int32_t *rows, void *stream)
+{
+    if (!inst || !rows) return fail(PP_EINVAL, "null pointer");
+    if (batch <= 0) return PP_OK;
+    DpGeom g;
+    if (!dp_geometry(inst, max_budget, &g, batch)) return fail(PP_EINVAL, "max_budget out of range");
+    if (inst->n == 0) {
+        for (int32_t b = 0; b < batch; ++b) rows[b] = 0;
+        return PP_OK;
+    }
+    if (!workspace) return fail(PP_EINVAL, "null workspace");
+    const DpWork w = dp_work_split(const_cast<uint32_t *>(workspace), batch, inst->n, g.words);
+    PP_CUDA(cudaMemcpyAsync(rows, w.nkept, sizeof(int32_t) * batch, cudaMemcpyDeviceToHost, (cudaStream_t)stream));
+    PP_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+    return PP_OK;
 }
