@@ -17,8 +17,9 @@ k = 4,096 slots, 16 starts, 6 rounds), inputs resident in HBM.
 
 --impl reference runs the oracle (the only reference implementation of this
 path) on the host cores and prints the same line with "impl": "reference".
-Multi-GPU (torchrun): each rank plans its own starts (weak scaling); the
-candidates are compared once after the timed region.
+Multi-GPU (torchrun): weak scaling, 16 starts per GPU out of 16 x N default
+start orders; rank r plans the starts s with s % N == r and the candidates
+are compared once after the timed region (no exchange while planning).
 """
 from __future__ import annotations
 
@@ -201,9 +202,15 @@ def run_native(args):
 
     inst = wl.make(BENCH_CONFIG)
     S, R = inst.starts, inst.rounds
-    orders = None if rank == 0 else wl.random_orders(inst.W, S, seed=1000 + rank)
     stream = torch.cuda.current_stream()
     ppi = pp.Instance.from_workload(inst)
+    orders = None
+    if world > 1:
+        # weak scaling: S starts per GPU out of S * world default orders, the
+        # same on every rank; rank r plans the starts s with s % world == r
+        from paper_2608_01655_gb300 import shard
+        all_orders = pp.pp_default_orders(ppi, S * world)
+        orders = all_orders[shard.my_starts(S * world, rank, world)]
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")   # 2x the 129 MB L2
 
     def barrier():
@@ -322,13 +329,11 @@ def run_native(args):
     e2e_value = world * cells_per_plan * args.steps / e2e_total
 
     # ---- candidates of all ranks compared once (outside the timed region) ---
-    best_obj, best_rank = res.objective, 0
+    best_obj, best_start = res.objective, res.best_start
     if world > 1:
-        t = torch.tensor([res.objective, -rank], dtype=torch.int64, device="cuda")
-        gathered = [torch.zeros_like(t) for _ in range(world)]
-        torch.distributed.all_gather(gathered, t)
-        cands = [(int(x[0]), -int(x[1])) for x in gathered]
-        best_obj, best_rank = max(cands, key=lambda c: (c[0], -c[1]))
+        mine = shard.my_starts(S * world, rank, world)
+        won = shard.exchange(res.objective, int(mine[res.best_start]), res.placement)
+        best_obj, best_start = won.objective, won.best_start
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -352,7 +357,7 @@ def run_native(args):
                     "ms_per_step": 1000 * e2e_total / args.steps},
             "gpu_launches": launches_per_plan * args.steps,
             "clocks": clocks,
-            "plan": {"objective": best_obj, "best_rank": best_rank, "best_start": res.best_start,
+            "plan": {"objective": best_obj, "best_start": best_start,
                      "dp_count": res.dp_count, "dp_cells": cells_per_plan,
                      "dp_rows_swept": phased.dp_rows_swept, "dp_cells_swept": phased.dp_rows_swept * k,
                      "sweeps": res.per_start_sweeps.tolist(),

@@ -316,6 +316,17 @@ pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_bud
 pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
                      int32_t no_prune);
 
+/*
+ * pp_default_orders -- the start orders pp_plan_run uses when it is given
+ * orders = NULL (Section IV-C: standalone-score order, its reverse, then
+ * SplitMix64 shuffles; the identity for one start), written to host
+ * [n_starts][W].  Runs the standalone-score DPs on the device when
+ * n_starts > 1.  Lets several processes split the starts of one plan: each
+ * computes the same orders and runs its share with pp_plan_run.
+ * Synchronous.  Errors: PP_EINVAL, PP_ENOMEM, PP_ECUDA.
+ */
+pp_status pp_default_orders(pp_instance *inst, int32_t n_starts, int32_t *orders, void *stream);
+
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);
 

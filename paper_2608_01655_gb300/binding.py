@@ -64,6 +64,7 @@ _SIGS = {
     "pp_tune_dp": [_i32, _i32, _i32, _i32],
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
     "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
+    "pp_default_orders": [_P, _i32, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -280,3 +281,10 @@ def pp_tune_dp(cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: b
                no_prune: bool = False):
     _check(_lib.pp_tune_dp(int(cluster_ctas), int(columns_per_thread), int(bool(force_flat)),
                            int(bool(no_prune))))
+
+
+def pp_default_orders(inst: Instance, n_starts: int, stream=None) -> np.ndarray:
+    """The start orders pp_plan_run uses when given none: [n_starts][W] int32."""
+    out = np.zeros((int(n_starts), inst.W), np.int32)
+    _check(_lib.pp_default_orders(inst.handle, int(n_starts), _host(out), _stream(stream)))
+    return out

@@ -82,7 +82,7 @@ static pp_status plan_buffers(pp_instance *inst, int B, PlanBuffers *pb)
 
 static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t R,
                            uint8_t *placement, int64_t *objective, pp_plan_stats *stats,
-                           cudaStream_t st)
+                           cudaStream_t st, bool orders_only = false)
 {
     const int32_t n = inst->n, W = inst->W;
     int launches = 0;
@@ -156,6 +156,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         }
     }
     if (stats && stats->orders_used) std::memcpy(stats->orders_used, ord.data(), sizeof(int32_t) * ord.size());
+    if (orders_only) return PP_OK;
 
     // ---- per-step worker / budget tables: work[t][s] = pi_s[t] -------------
     std::vector<int32_t> hw((size_t)W * B, 0), hk((size_t)W * B, 0);
@@ -303,6 +304,19 @@ extern "C" pp_status pp_plan_run(pp_instance *inst, int32_t n_starts, const int3
     if (!objective || (inst->n > 0 && !placement)) return fail(PP_EINVAL, "null output pointer");
     cudaStream_t st = (cudaStream_t)stream;
     pp_status s = plan_impl(inst, n_starts, orders, max_rounds, placement, objective, stats, st);
+    if (s != PP_OK) return s;
+    return pp_instance_sync(inst, stream);
+}
+
+extern "C" pp_status pp_default_orders(pp_instance *inst, int32_t n_starts, int32_t *orders, void *stream)
+{
+    if (!inst) return fail(PP_EINVAL, "null instance");
+    if (n_starts < 1) return fail(PP_EINVAL, "n_starts must be >= 1");
+    if (!orders) return fail(PP_EINVAL, "null output pointer");
+    pp_plan_stats st = {};
+    st.orders_used = orders;
+    int64_t unused = 0;
+    pp_status s = plan_impl(inst, n_starts, nullptr, 0, nullptr, &unused, &st, (cudaStream_t)stream, true);
     if (s != PP_OK) return s;
     return pp_instance_sync(inst, stream);
 }

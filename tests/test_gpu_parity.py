@@ -324,3 +324,14 @@ def test_bounded_wait_reports_timeout(pp, oracle_lib):
     ob, oc = oracle_lib.rooted_dp(inst.parent, inst.weight, profits[0], k)
     assert best[0] == ob
     np.testing.assert_array_equal(chosen[0], oc)
+
+
+def test_default_orders_match_oracle(pp, oracle_lib):
+    """pp_default_orders (used to split starts across processes) equals the
+    oracle's start orders: standalone-score order, reverse, SplitMix64 shuffles."""
+    for cfg in (0, 1):
+        inst = wl.make(cfg)
+        with pp.Instance.from_workload(inst) as ppi:
+            for S in (1, 2, 7):
+                np.testing.assert_array_equal(pp.pp_default_orders(ppi, S),
+                                              oracle_lib.default_orders(oracle_lib.Problem.from_instance(inst), S))
