@@ -42,6 +42,7 @@ METRIC = "tree-DP cell-updates/s and end-to-end plan time (n=50k, 16 workers) vs
 UNIT = "cell-updates/s"
 BENCH_CONFIG = 3            # the n = 50,000 / W = 16 / k = 4,096 workload
 SM_COUNT = 152
+INT32_LANES_PER_SM = 64     # integer add/compare/select/logic: 16 lanes per scheduler, 4 schedulers
 ALU_OPS_PER_CELL = 6        # int64 add, compare, select = 2 + 2 + 2 int32 lane operations
 
 
@@ -281,7 +282,7 @@ def run_native(args):
     cells_swept = rows_swept * k
     peaks, peak_kind = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
-    alu_peak = SM_COUNT * 4 * 32 * sm_mhz * 1e6 / ALU_OPS_PER_CELL      # cells/s, issue-bound
+    alu_peak = SM_COUNT * INT32_LANES_PER_SM * sm_mhz * 1e6 / ALU_OPS_PER_CELL   # cells/s
     achieved = cells_swept / dp_t                 # cells the kernel actually computed
     # algorithmic bytes of one launch: decision bits + p/w/next + skip-row pushes
     order, nxt, skipc, pushl, depth = pp.pp_row_plan(inst.parent)
@@ -293,8 +294,8 @@ def run_native(args):
         traffic = tr["bytes_per_launch"] * cells_launch / tr["cells_per_launch"]
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": alu_peak / 1e12, "unit": "Tcell/s",
                 "frac": achieved / alu_peak, "traffic": traffic,
-                "peak_source": f"derived: {SM_COUNT} SMs x 4 SMSP x 32 lanes x {sm_mhz:.0f} MHz / "
-                               f"{ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
+                "peak_source": f"derived: {SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 ALU lanes x "
+                               f"{sm_mhz:.0f} MHz / {ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
                 "kernel": "k_tree_dp_wave", "launch_ms": 1000 * dp_t, "cells_per_launch": cells_launch,
                 "cells_swept_per_launch": cells_swept, "rows_swept_per_launch": rows_swept,
                 "hbm_bmin_gbs": bmin / dp_t / 1e9,
