@@ -5,6 +5,8 @@ formula: they compare against exhaustive enumeration, against the more
 primitive materialisation rule of Section III-A, against closed forms
 (Theorem 2's spider) or against theorems (Lemma 1, Prop. 1, Theorem 3).
 """
+import os
+
 import numpy as np
 import pytest
 
@@ -143,12 +145,27 @@ def test_lemma1_reduction(oracle_lib):
             oracle_lib.objective_Fpair(_prob(oracle_lib, src), pl)
 
 
+def _golden(name):
+    """Key -> value tokens of a fixture under tests/golden/ ('#' starts a comment)."""
+    out = {}
+    for line in open(os.path.join(os.path.dirname(__file__), "golden", name)):
+        line = line.split("#", 1)[0].split()
+        if line:
+            out[line[0]] = line[1:]
+    return out
+
+
 def test_theorem2_spider_closed_form(oracle_lib):
     """Theorem 2's spider: covering the first x_i chunks of leg i saves
-    lambda_i * sum_{d<=x_i}(2d - 1) = x_i^2 / s_i; demand scaled by L = lcm(s_i)."""
-    s = [3, 4, 5, 4, 3, 5]                      # a 3-Partition instance, B = 12, q = 2
+    lambda_i * sum_{d<=x_i}(2d - 1) = x_i^2 / s_i; demand scaled by L = lcm(s_i).
+    The instance and its optimum L*q*B are the fixture tests/golden/spider_3partition.txt."""
+    g = _golden("spider_3partition.txt")
+    s = [int(v) for v in g["legs"]]             # a 3-Partition instance
+    q, B = int(g["q"][0]), int(g["B"][0])
+    assign = [int(v) for v in g["assignment"]]
+    optimum = int(g["optimum"][0])
     L = int(np.lcm.reduce(s))
-    q, B = 2, 12
+    assert L * q * B == optimum
     n = sum(s)
     parent, depth, leg = [], [], []
     for i, si in enumerate(s):
@@ -177,11 +194,12 @@ def test_theorem2_spider_closed_form(oracle_lib):
                     pl[int(rng.integers(q)), b] = 1       # any holder covers it
             expect = sum(L * xi * xi // si for xi, si in zip(x, s))
             assert oracle_lib.objective(prob, pl) == expect
-        # a valid 3-partition ({3,4,5}, {4,3,5}) reaches L * q * B
+            assert expect <= optimum
+        # the fixture's valid 3-partition reaches the optimum
         pl = np.zeros((W, n), np.uint8)
         for b in range(n):
-            pl[0 if leg[b] < 3 else 1, b] = 1
-        assert oracle_lib.objective(prob, pl) == L * q * B
+            pl[assign[leg[b]], b] = 1
+        assert oracle_lib.objective(prob, pl) == optimum
 
 
 # ------------------------------------------------------------- marginals ---
@@ -275,21 +293,24 @@ def test_default_orders_shape(oracle_lib):
 
 # ------------------------------------------------- generator constants ---
 def test_generator_constants_match_paper_arithmetic():
-    """Fig. 1, Table I and RQ1 arithmetic that the cost generator is built on."""
-    assert wl.CHUNK_BYTES == 18_874_368                              # "18.9-MB"
-    assert round(wl.CHUNK_BYTES / 1e6, 1) == 18.9
-    t = int(wl.fetch_us(wl.CHUNK_BYTES, 1_500_000_000))              # "about 100.7 ms"
-    assert t == 100_663 and round(t / 1000, 1) == 100.7
-    b7 = 512 * 57_344                                                 # L4/A100-7B, "29.4-MB"
-    assert round(b7 / 1e6, 1) == 29.4
-    assert round(512 * 262_144 / 1e6, 1) == 134.2                    # A100-32B, "134.2-MB"
+    """Fig. 1 and RQ1 figures (fixture tests/golden/paper_constants.txt) that
+    the cost generator is built on, recomputed from its constants and compared
+    at the printed precision."""
+    g = {k: float(v[0]) for k, v in _golden("paper_constants.txt").items()}
+    assert wl.CHUNK_BYTES == 512 * 36_864                             # 3B: 36,864 B per token
+    assert round(wl.CHUNK_BYTES / 1e6, 1) == g["kv_bytes_3b_chunk_mb"]
+    t = int(wl.fetch_us(wl.CHUNK_BYTES, 1_500_000_000))
+    assert round(t / 1000, 1) == g["fetch_3b_at_1p5gbps_ms"]
+    b7 = 512 * 57_344                                                 # 7B: 57,344 B per token
+    assert round(b7 / 1e6, 1) == g["kv_bytes_7b_chunk_mb"]
+    assert round(512 * 262_144 / 1e6, 1) == g["kv_bytes_32b_chunk_mb"]
     f7 = int(wl.fetch_us(b7, 3_000_000_000)) / 1000                   # ms at 3 Gb/s
-    p_cross = (f7 - 48.1) / 0.0050                                    # A100-7B fit
-    assert abs(p_cross - 6100) / 6100 < 0.02                          # "near 6.1K tokens"
-    assert 170.2 > f7                                                 # L4-7B "favors fetching"
-    # the middle generator class crosses the 1.5 Gb/s fetch near 3.8K tokens (Fig. 1, L4)
+    p_cross = (f7 - g["a100_7b_fit_base_ms"]) / g["a100_7b_fit_slope_ms"]
+    assert abs(p_cross - g["a100_7b_crossover_tokens"]) / g["a100_7b_crossover_tokens"] < 0.02
+    assert g["l4_7b_fit_base_ms"] > f7                                # L4-7B favors fetching
+    # the middle generator class crosses the 1.5 Gb/s fetch near the L4 crossover
     p_mid = (t - wl.BETA_US[1]) / wl.ALPHA_US_PER_TOKEN[1]
-    assert abs(p_mid - 3800) < 100
+    assert abs(p_mid - g["l4_crossover_tokens"]) < 100
     assert wl.ALPHA_US_PER_TOKEN[1] == 3 * wl.ALPHA_US_PER_TOKEN[0]
     assert wl.ALPHA_US_PER_TOKEN[2] == 8 * wl.ALPHA_US_PER_TOKEN[0]
 
