@@ -174,16 +174,26 @@ def _dist():
     return world, rank, local
 
 
+TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "tree_dp_traffic_paper-n50000-W16-k4096.md")
+DP_SOURCES = [os.path.join(ROOT, "paper_2608_01655_gb300", "csrc", f) for f in ("pp_dp.cu", "pp_internal.cuh")]
+
+
+def dp_source_sha256():
+    h = hashlib.sha256()
+    for f in DP_SOURCES:
+        h.update(open(f, "rb").read())
+    return h.hexdigest()
+
+
 def _traffic_record():
-    """Per-launch DRAM traffic of the DP kernel from a committed ncu summary,
-    valid only while the kernel source is unchanged."""
-    path = os.path.join(ROOT, "profiles", "tree_dp_traffic.json")
-    src = os.path.join(ROOT, "paper_2608_01655_gb300", "csrc", "pp_dp.cu")
+    """Per-launch DRAM traffic of the tree-DP launch from the committed ncu
+    summary (its `traffic_record:` line), used only while the DP sources are
+    unchanged since the counters were taken."""
     try:
-        rec = json.load(open(path))
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
-        if rec.get("kernel_src_sha256") == sha:
-            return rec
+        for line in open(TRAFFIC_SUMMARY):
+            if line.startswith("traffic_record:"):
+                rec = json.loads(line.split(":", 1)[1])
+                return rec if rec.get("kernel_src_sha256") == dp_source_sha256() else None
     except (OSError, ValueError):
         pass
     return None
@@ -223,7 +233,7 @@ def run_native(args):
         res = pp.pp_plan_run(ppi, S, orders, R)
     cells_per_plan = res.dp_cells
     launches_per_plan = res.kernel_launches
-    times = []
+    times, phase_sum = [], [0.0, 0.0, 0.0]
     with ClockSampler(local) as clk:
         for _ in range(args.steps):
             flush.fill_(1)
@@ -232,11 +242,14 @@ def run_native(args):
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            res = pp.pp_plan_run(ppi, S, orders, R)
+            # events around every launch of the plan (read after the plan returns)
+            res = pp.pp_plan_run(ppi, S, orders, R, time_phases=True)
             e1.record(stream)
             torch.cuda.synchronize()
             barrier()
             times.append(e0.elapsed_time(e1) / 1000.0)
+            for x in range(3):
+                phase_sum[x] += res.phase_ms[x]
     clocks = clk.summary()
     total = sum(times)
     if world > 1:
@@ -245,59 +258,37 @@ def run_native(args):
         total = float(t.item())
     value = world * cells_per_plan * args.steps / total
 
-    # ---- per-phase device time of one plan (events around every launch) ----
-    phased = pp.pp_plan_run(ppi, S, orders, R, time_phases=True)
-
-    # ---- the dominant kernel, timed live: the plan's DP launch (S items) ----
+    # ---- the dominant kernel: the plan's batched tree-DP launches (row pruning
+    # + Eq. 9 sweep), CUDA events on the launching stream over the timed region
     k = int(inst.budget.max())
     n = inst.n
-    masks = np.zeros((S, n), np.uint32)
-    for m in range(inst.W):
-        masks |= res.placement[m].astype(np.uint32) << np.uint32(m)
-    masks_t = torch.from_numpy(masks.view(np.int32)).cuda()
-    workers = torch.arange(S, dtype=torch.int32, device="cuda") % inst.W
-    prof = torch.zeros((S, n), dtype=torch.int64, device="cuda")
-    pp.pp_marginals(ppi, workers, masks_t, prof)
-    bud = torch.full((S,), k, dtype=torch.int32, device="cuda")
-    best = torch.zeros(S, dtype=torch.int64, device="cuda")
-    bits = torch.zeros(pp.pp_dp_bits_size(ppi, S, k) // 4, dtype=torch.int32, device="cuda")
-    dp_times, mg_times = [], []
-    for it in range(args.warmup + args.probe_iters):
-        flush.fill_(2)
-        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-        e[0].record(stream)
-        pp.pp_marginals(ppi, workers, masks_t, prof)
-        e[1].record(stream)
-        e[2].record(stream)
-        pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
-        e[3].record(stream)
-        torch.cuda.synchronize()
-        if it >= args.warmup:
-            mg_times.append(e[0].elapsed_time(e[1]) / 1000.0)
-            dp_times.append(e[2].elapsed_time(e[3]) / 1000.0)
-    ppi.sync()
-    dp_t = statistics.mean(dp_times)
-    cells_launch = S * n * k
-    rows_swept = int(pp.pp_dp_rows_swept(ppi, S, k, bits).sum())
+    nl = res.dp_launches
+    dp_t = phase_sum[1] / 1000.0 / (nl * args.steps)              # s per launch
+    items = res.dp_count / nl                                      # DPs per launch
+    cells_launch = res.dp_cells / nl                               # n x k table cells per launch
+    rows_swept = res.dp_rows_swept / nl                            # kept rows per launch
     cells_swept = rows_swept * k
     peaks, peak_kind = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = SM_COUNT * INT32_LANES_PER_SM * sm_mhz * 1e6 / ALU_OPS_PER_CELL   # cells/s
     achieved = cells_swept / dp_t                 # cells the kernel actually computed
-    # algorithmic bytes of one launch: decision bits + p/w/next + skip-row pushes
+    # algorithmic bytes of one launch: decision bits of the swept rows + p/w/next
+    # of every row + skip-row pushes
     order, nxt, skipc, pushl, depth = pp.pp_row_plan(inst.parent)
     pushes = int((pushl >= 0).sum())
-    bmin = S * (n * (k + 1) / 8 + 16 * n + 16 * (k + 1) * pushes)
+    bmin = rows_swept * (k + 1) / 8 + items * (16 * n + 16 * (k + 1) * pushes)
     tr = _traffic_record()
     traffic = None
-    if tr and tr.get("cells_per_launch"):
-        traffic = tr["bytes_per_launch"] * cells_launch / tr["cells_per_launch"]
+    if tr and tr.get("cells_swept_per_launch"):
+        traffic = tr["bytes_per_launch"] * cells_swept / tr["cells_swept_per_launch"]
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": alu_peak / 1e12, "unit": "Tcell/s",
                 "frac": achieved / alu_peak, "traffic": traffic,
                 "peak_source": f"derived: {SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 ALU lanes x "
                                f"{sm_mhz:.0f} MHz / {ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
-                "kernel": "k_tree_dp_wave", "launch_ms": 1000 * dp_t, "cells_per_launch": cells_launch,
-                "cells_swept_per_launch": cells_swept, "rows_swept_per_launch": rows_swept,
+                "kernel": "k_prune + k_tree_dp_wave (one batched tree-DP launch of the plan)",
+                "launches": nl * args.steps, "launch_ms": 1000 * dp_t, "items_per_launch": items,
+                "cells_per_launch": cells_launch, "cells_swept_per_launch": cells_swept,
+                "rows_swept_per_launch": rows_swept,
                 "hbm_bmin_gbs": bmin / dp_t / 1e9,
                 "hbm_bmin_frac": bmin / dp_t / 1e9 / float(peaks.get("hbm_gbs", 6800.0)),
                 "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0)), "hbm_peak_kind": peak_kind}
@@ -360,12 +351,12 @@ def run_native(args):
             "clocks": clocks,
             "plan": {"objective": best_obj, "best_start": best_start,
                      "dp_count": res.dp_count, "dp_cells": cells_per_plan,
-                     "dp_rows_swept": phased.dp_rows_swept, "dp_cells_swept": phased.dp_rows_swept * k,
+                     "dp_launches": nl, "dp_rows_swept": res.dp_rows_swept,
+                     "dp_cells_swept": res.dp_rows_swept * k,
                      "sweeps": res.per_start_sweeps.tolist(),
                      "step_ms": [round(1000 * t, 3) for t in times]},
-            "marginals_launch_ms": 1000 * statistics.mean(mg_times),
-            "phase_ms": {"marginals": phased.phase_ms[0], "tree_dp": phased.phase_ms[1],
-                         "traceback_accept": phased.phase_ms[2]},
+            "phase_ms": {"marginals": phase_sum[0] / args.steps, "tree_dp": phase_sum[1] / args.steps,
+                         "traceback_accept": phase_sum[2] / args.steps},
             "dp_geometry": pp.pp_dp_geometry(ppi, S, k),
         }
         print(json.dumps(line), flush=True)
@@ -405,7 +396,6 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
-    ap.add_argument("--probe-iters", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-dp", type=int, default=0, metavar="B",
                     help="only launch the tree DP of B items twice (a small case for ncu) and exit")

@@ -71,6 +71,7 @@ typedef struct {
     float phase_ms[3];             /* out (if time_phases): device time of the marginal,
                                       tree-DP (with its row pruning) and traceback launches,
                                       summed over the plan */
+    int32_t dp_launches;           /* out: batched tree-DP launches (one per plan step) */
 } pp_plan_stats;
 
 /*

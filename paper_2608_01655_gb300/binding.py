@@ -44,7 +44,7 @@ class PlanStats(ctypes.Structure):
     _fields_ = [("per_start_objective", _P), ("per_start_sweeps", _P), ("per_start_accepted", _P),
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
                 ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
-                ("phase_ms", ctypes.c_float * 3)]
+                ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32)]
 
 
 _SIGS = {
@@ -237,6 +237,7 @@ class PlanResult:
     kernel_launches: int
     phase_ms: tuple = ()
     dp_rows_swept: int = 0
+    dp_launches: int = 0
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
@@ -260,7 +261,8 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                             ctypes.byref(st), _stream(stream)))
     return PlanResult(placement[:, :n].copy(), int(obj.value), int(st.best_start), per, sw, acc, used,
                       int(st.dp_count), int(st.dp_cells), int(st.kernel_launches),
-                      tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept))
+                      tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept),
+                      int(st.dp_launches))
 
 
 def pp_test_inject(kind: int, value: int):

@@ -113,7 +113,7 @@ __device__ __forceinline__ void st_relaxed_cluster_u64_if(bool pred, uint32_t ad
 {
     asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %0, 0;\n\t"
                  "@p st.relaxed.cluster.shared::cluster.u64 [%1], %2;\n\t}"
-                 ::"r"((uint32_t)pred), "r"(addr), "l"(v) : "memory");
+                 ::"r"((uint32_t)pred), "r"(addr), "l"(v));
 }
 __device__ __forceinline__ void ld_volatile_v2_u64(const uint64_t *p, uint64_t &a, uint64_t &b)
 {
@@ -372,10 +372,13 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
                 }
             }
             const uint32_t mbase = 1u << (sb * kSub);
+            int4 mmv[kSub];
+#pragma unroll
+            for (int u = 0; u < kSub; ++u) mmv[u] = my_meta[sb * kSub + u];
             // one row of Eq. 9 for this warp's columns; STACK: the row may push or pop
             auto row = [&](const int u, const bool STACK) {
                 const int r = r0 + u;
-                const int4 mm = my_meta[sb * kSub + u];
+                const int4 mm = mmv[u];
                 const int64_t p = (int64_t)(((uint64_t)(uint32_t)mm.y << 32) | (uint32_t)mm.x);
                 const int32_t m = mm.z;
                 // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
@@ -646,7 +649,7 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 __global__ void __launch_bounds__(256)
 k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
-            const int32_t *__restrict__ wpre, uint8_t *__restrict__ chosen, AcceptArgs acc)
+            uint8_t *__restrict__ chosen, AcceptArgs acc)
 {
     const int item = blockIdx.x;
     uint32_t hbit = 0;
@@ -659,7 +662,8 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
         if (h < 0 || h >= 32) return;
         hbit = 1u << h;
         M = acc.mask + (size_t)item * n;
-        for (int32_t x = threadIdx.x; x < n; x += blockDim.x) M[x] &= ~hbit;
+        // fire-and-forget reductions: no thread waits for the old mask words
+        for (int32_t x = threadIdx.x; x < n; x += blockDim.x) atomicAnd(M + x, ~hbit);
     } else {
         uint8_t *ch = chosen + (size_t)item * n;
         for (int32_t x = threadIdx.x; x < n; x += blockDim.x) ch[x] = 0;
@@ -699,7 +703,7 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
         const bool take = live && col > 0 && bit(row, col);
         const int pos = live ? rl[row] : -1;
         const int s1 = live ? sk[row] : -1, s2 = live ? sk2[row] : -1;
-        const int wrow = live ? wpre[pos] : 0;
+        const int wrow = live ? (unit_weights ? 1 : ws[row] - ws[row + 1]) : 0;   // w of kept row `row`
         const uint32_t tm = __ballot_sync(kFull, take);
         int h0;                                           // the half that continues the walk
         if (tm & 1u) {
@@ -717,7 +721,7 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
         const uint32_t run = (tm >> (16 * h0)) & 0xFFFFu;
         const int l0 = __ffs(~run) - 1 < 16 ? __ffs(~run) - 1 : 16;   // first lane of the half not taken
         if (half == h0 && l < l0) {
-            if (M) M[pos] |= hbit;
+            if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
             else chosen[(size_t)item * n + order[pos]] = 1;
         }
         const int src = 16 * h0 + (l0 < 16 ? l0 : 15);
@@ -781,7 +785,7 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int *total, int *sh)
 template <bool BYNODE>
 __global__ void __launch_bounds__(1024)
 k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
-        const int32_t *__restrict__ next, const int32_t *__restrict__ ppos,
+        const int32_t *__restrict__ next, const int2 *__restrict__ pspan,
         const int32_t *__restrict__ wpre, const int32_t *__restrict__ item_active, DpWork w,
         int prune, unsigned long long *__restrict__ rows_kept)
 {
@@ -806,22 +810,25 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
     }
     if (t == 0) cnt[n] = total;
     __syncthreads();
-    // kept rows in sweep order r = n - 1 - i
-    auto keep = [&](int i) -> bool {
-        if (!prune) return true;
-        const int pa = ppos[i];
-        return pa < 0 || cnt[next[pa]] - cnt[pa + 1] > 0;
-    };
+    // kept rows in sweep order r = n - 1 - i; the flag goes to kx[i] first
+    // (0 kept, -1 dropped) and is replaced by the kept index below
     int kc = 0;
-    for (int r = lo; r < hi; ++r) kc += keep(n - 1 - r);
+    for (int r = lo; r < hi; ++r) {
+        const int i = n - 1 - r;
+        bool kp = true;
+        if (prune) {
+            const int2 sp = pspan[i];
+            kp = sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0;
+        }
+        kx[i] = kp ? 0 : -1;
+        kc += kp;
+    }
     int kex = block_exclusive_scan(kc, &total, sh);
     for (int r = lo; r < hi; ++r) {
         const int i = n - 1 - r;
-        if (keep(i)) {
+        if (kx[i] == 0) {
             rl[kex] = i;
             kx[i] = kex++;
-        } else {
-            kx[i] = -1;
         }
     }
     const int nk = total;
@@ -1031,10 +1038,10 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
 {
     // the pruned sweep of every item, then the DP over its kept rows
     if (by_node)
-        k_prune<true><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_ppos,
+        k_prune<true><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
                                               inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
     else
-        k_prune<false><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_ppos,
+        k_prune<false><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
                                                inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
     PP_CUDA(cudaGetLastError());
     uint32_t *bits = work.bits;
@@ -1104,7 +1111,7 @@ pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, con
     AcceptArgs a;
     if (acc) a = *acc;
     k_traceback<<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
-                                       inst->d_order, inst->d_wpre, chosen, a);
+                                       inst->d_order, chosen, a);
     PP_CUDA(cudaGetLastError());
     return PP_OK;
 }

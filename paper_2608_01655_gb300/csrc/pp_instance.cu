@@ -215,7 +215,7 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     cudaFree(inst->d_wpre);
     cudaFree(inst->d_meta);
     cudaFree(inst->d_wave);
-    cudaFree(inst->d_ppos);
+    cudaFree(inst->d_pspan);
     cudaFree(inst->d_budget);
     cudaFree(inst->d_a);
     cudaFree(inst->d_delta);
@@ -293,13 +293,16 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if ((s = upload(&inst->d_meta, inst->h_meta.data(), n, st))) return s;
     if ((s = upload(&inst->d_wave, inst->h_wave.data(), n, st))) return s;
     {
-        std::vector<int32_t> pos(n), ppos(n);
+        // for the parent x of each position: the preorder range [x + 1, next(x))
+        // of x's strict descendants (the pruned sweep's test)
+        std::vector<int32_t> pos(n);
+        std::vector<int2> span(n);
         for (int32_t i = 0; i < n; ++i) pos[inst->h_order[i]] = i;
         for (int32_t i = 0; i < n; ++i) {
             const int32_t par = parent[inst->h_order[i]];
-            ppos[i] = par < 0 ? -1 : pos[par];
+            span[i] = par < 0 ? make_int2(-1, -1) : make_int2(pos[par] + 1, inst->h_next[pos[par]]);
         }
-        if ((s = upload(&inst->d_ppos, ppos.data(), n, st))) return s;
+        if ((s = upload(&inst->d_pspan, span.data(), n, st))) return s;
         PP_CUDA(cudaStreamSynchronize(st));          // the host vectors die here
     }
     if ((s = upload(&inst->d_budget, budget, W, st))) return s;

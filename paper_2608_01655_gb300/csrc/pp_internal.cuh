@@ -123,7 +123,7 @@ struct pp_instance {
     int32_t *d_wpre = nullptr;          // [n] chunk weight
     int32_t *d_meta = nullptr;          // [n] packed skip / push codes
     int32_t *d_wave = nullptr;          // [n] wavefront-kernel row metadata
-    int32_t *d_ppos = nullptr;          // [n] preorder position of the parent, -1 for roots
+    int2 *d_pspan = nullptr;            // [n] parent x's strict-descendant range (x+1, next(x)); roots -1
     int32_t *d_budget = nullptr;        // [W]
     int64_t *d_a = nullptr;             // mode 0: [W][n] a_m(b)       (Eq. 2)
     int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)

@@ -108,6 +108,22 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
     unsigned long long *rows_kept = pb.rows;
     PP_CUDA(cudaMemsetAsync(rows_kept, 0, sizeof(unsigned long long), st));
 
+    // optional per-phase timing: events around every launch, read once at the end
+    const bool timing = stats && stats->time_phases;
+    int32_t dp_launches = 0;
+    struct Events {
+        std::vector<cudaEvent_t> v;
+        ~Events() { for (cudaEvent_t e : v) cudaEventDestroy(e); }
+    } ev;
+    auto mark = [&]() -> pp_status {
+        if (!timing) return PP_OK;
+        cudaEvent_t e;
+        PP_CUDA(cudaEventCreate(&e));
+        ev.v.push_back(e);
+        PP_CUDA(cudaEventRecord(e, st));
+        return PP_OK;
+    };
+
     // ---- start orders -----------------------------------------------------
     std::vector<int32_t> ord((size_t)S * W);
     if (orders) {
@@ -131,11 +147,16 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
             PP_CUDA(cudaMemcpyAsync(d_ids, ids.data(), 4 * W, cudaMemcpyHostToDevice, st));
             PP_CUDA(cudaMemcpyAsync(d_kb, kb.data(), 4 * W, cudaMemcpyHostToDevice, st));
             PP_CUDA(cudaMemsetAsync(pb.mask, 0, (size_t)4 * std::max(n, 1) * W, st));
+            if ((s = mark())) return s;
             if ((s = launch_marginals(inst, W, d_ids, pb.mask, false, nullptr, pb.profit, nullptr, st))) return s;
+            if ((s = mark())) return s;
             if ((s = launch_tree_dp(inst, W, pb.profit, false, d_kb, nullptr, gw, pb.best, work_w, st, maxk,
                                     rows_kept)))
                 return s;
+            if ((s = mark())) return s;
+            if ((s = mark())) return s;   // no traceback for the standalone scores
             launches += 3;
+            dp_launches += 1;
             std::vector<int64_t> score(W);
             standalone_cells = (int64_t)n * sumk;
             PP_CUDA(cudaMemcpyAsync(score.data(), pb.best, 8 * W, cudaMemcpyDeviceToHost, st));
@@ -176,17 +197,6 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
 
     int dp_count = standalone_cells ? W : 0;
     int64_t cells = standalone_cells;
-    // optional per-phase timing: events around every launch, read once at the end
-    const bool timing = stats && stats->time_phases;
-    std::vector<cudaEvent_t> ev;
-    auto mark = [&]() -> pp_status {
-        if (!timing) return PP_OK;
-        cudaEvent_t e;
-        PP_CUDA(cudaEventCreate(&e));
-        PP_CUDA(cudaEventRecord(e, st));
-        ev.push_back(e);
-        return PP_OK;
-    };
     auto step = [&](int t, int greedy) -> pp_status {
         const int32_t *wk = pb.work + (size_t)t * B;
         const int32_t *kb = pb.kbud + (size_t)t * B;
@@ -209,6 +219,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         if ((r = launch_traceback(inst, S, work, g, kb, nullptr, &a, st))) return r;
         if ((r = mark())) return r;
         launches += 4;
+        dp_launches += 1;
         return PP_OK;
     };
 
@@ -275,18 +286,18 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         stats->dp_cells = cells;
         stats->kernel_launches = launches;
         stats->dp_rows_swept = (int64_t)rows_swept;
+        stats->dp_launches = dp_launches;
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
-        for (size_t x = 0; x + 3 < ev.size(); x += 4) {
+        for (size_t x = 0; x + 3 < ev.v.size(); x += 4) {
             float a = 0.f, b = 0.f, c = 0.f;
-            cudaEventElapsedTime(&a, ev[x], ev[x + 1]);
-            cudaEventElapsedTime(&b, ev[x + 1], ev[x + 2]);
-            cudaEventElapsedTime(&c, ev[x + 2], ev[x + 3]);
+            cudaEventElapsedTime(&a, ev.v[x], ev.v[x + 1]);
+            cudaEventElapsedTime(&b, ev.v[x + 1], ev.v[x + 2]);
+            cudaEventElapsedTime(&c, ev.v[x + 2], ev.v[x + 3]);
             stats->phase_ms[0] += a;
             stats->phase_ms[1] += b;
             stats->phase_ms[2] += c;
         }
     }
-    for (cudaEvent_t e : ev) cudaEventDestroy(e);
     return PP_OK;
 }
 
