@@ -367,8 +367,9 @@ def run_native(args):
 
 
 def run_profile_dp(args):
-    """A small case for ncu: marginals then the tree DP of `--profile-dp B`
-    items of the paper-scale workload, launched twice (ncu captures the second)."""
+    """A small case for ncu: marginals, the tree DP and the traceback of
+    `--profile-dp B` items of the paper-scale workload, launched twice (ncu
+    captures the second)."""
     import torch
     torch.cuda.set_device(0)
     from paper_2608_01655_gb300 import binding as pp
@@ -382,9 +383,11 @@ def run_profile_dp(args):
     bud = torch.full((B,), k, dtype=torch.int32, device="cuda")
     best = torch.zeros(B, dtype=torch.int64, device="cuda")
     bits = torch.zeros(pp.pp_dp_bits_size(ppi, B, k) // 4, dtype=torch.int32, device="cuda")
+    chosen = torch.zeros((B, n), dtype=torch.uint8, device="cuda")
     for _ in range(2):
         pp.pp_marginals(ppi, workers, masks, prof)
         pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
+        pp.pp_traceback(ppi, bits, bud, k, chosen)
     ppi.sync()
     print(json.dumps({"profile_dp": B, "geometry": pp.pp_dp_geometry(ppi, B, k), "best": best.tolist()}))
     return 0
@@ -398,7 +401,7 @@ def main():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-dp", type=int, default=0, metavar="B",
-                    help="only launch the tree DP of B items twice (a small case for ncu) and exit")
+                    help="only launch the tree DP and traceback of B items twice (a small case for ncu) and exit")
     args = ap.parse_args()
     if args.profile_dp:
         return run_profile_dp(args)

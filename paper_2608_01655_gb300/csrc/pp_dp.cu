@@ -220,9 +220,8 @@ constexpr uint64_t kLapBit = 1ull << 63;
 
 template <int C, int WMAX>
 __global__ void __launch_bounds__(512, 1)
-k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
-               const int32_t *__restrict__ nkept, const int64_t *__restrict__ profit,
-               const int32_t *__restrict__ order, const int32_t *__restrict__ wmeta,
+k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
+               const int32_t *__restrict__ rowm, const int32_t *__restrict__ nkept,
                const int32_t *__restrict__ item_budget, int32_t max_budget,
                const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
                uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
@@ -278,13 +277,14 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
     const bool publish = has_next && lane == 31 && g != g_drop_publish_warp;   // this lane stores
     const bool lane0 = lane == 0;
 
-    const int64_t *Pp = profit + (size_t)item * n;
     uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
-    int64_t *const my_stk = stk + threadIdx.x, *const my_gst = gst + threadIdx.x;
-    // the rows this item sweeps: all of them, or the kept rows of the pruned sweep
-    const int nrows = rowlist ? nkept[item] : n;
-    const int32_t *rows = rowlist ? rowlist + (size_t)item * n : nullptr;
+    int64_t *const my_gst = gst + threadIdx.x;
+    // the kept rows of the pruned sweep, with their profit and metadata
+    // gathered in sweep order
+    const int nrows = nkept[item];
+    const int64_t *Rp = rowp + (size_t)item * n;
+    const int32_t *Rm = rowm + (size_t)item * n;
     const int nblk_item = (nrows + 31) / 32;
 
     int64_t cur[C], top[C];
@@ -294,14 +294,14 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
         top[c] = 0;
     }
     // row metadata, 32 rows per block: lane l loads row blk*32 + l one block
-    // ahead and stages (p, m) in shared memory for the warp; rows past the
-    // last one are no-ops (p = -inf, skip = the row just computed), so every
-    // warp sweeps nblk_item * 32 rows
+    // ahead; the warp stages the profits (and stack levels) in shared memory
+    // and turns the flags into warp-uniform masks, bit = row of the block.
+    // Rows past the last one are no-ops (p = -inf, skip = the row just
+    // computed), so every warp sweeps nblk_item * 32 rows.
     auto load_meta = [&](int r, int64_t &pv, int32_t &mv) {
         if (r < nrows) {
-            const int i = rows ? rows[r] : n - 1 - r;
-            pv = Pp[order ? order[i] : i];
-            mv = wmeta[i];
+            pv = Rp[r];         // one independent load each: nothing waits
+            mv = Rm[r];         // for them before the next block
         } else {
             pv = kNeg;
             mv = 0;
@@ -315,12 +315,22 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
     int64_t carry[WMAX];
 #pragma unroll
     for (int q = 0; q < WMAX; ++q) carry[q] = has_prev ? 0 : (q == WMAX - 1 ? 0 : kNeg);
+    int64_t *const my_p = reinterpret_cast<int64_t *>(my_meta);     // [32] profits of the block
+    int32_t *const my_lv = reinterpret_cast<int32_t *>(my_p + 32);  // [32] stack levels
 
     for (int blk = 0; blk < nblk_item && !aborted; ++blk) {
         __syncwarp();
-        my_meta[lane] = make_int4((int)(uint32_t)pnext, (int)(uint32_t)((uint64_t)pnext >> 32), mnext,
-                                  (mnext & (3 << 3)) == (kWaveCur << 3));
-        const uint32_t stack_rows = __ballot_sync(kFull, (mnext & kWaveStackOps) != 0);   // bit = row of the block
+        my_p[lane] = pnext;
+        my_lv[lane] = (int32_t)((uint32_t)mnext >> 16);
+        const uint32_t cur_rows = __ballot_sync(kFull, (mnext & (3 << 3)) == (kWaveCur << 3));
+        const uint32_t push_rows = __ballot_sync(kFull, (mnext & kWavePush) != 0);
+        const uint32_t reload_rows = __ballot_sync(kFull, (mnext & kWaveReload) != 0);
+        const uint32_t zero_rows = __ballot_sync(kFull, (mnext & kWaveZeroTop) != 0);
+        uint32_t w1_rows = 0, w2_rows = 0;          // bits 0 and 1 of w - 1 (weights <= 4)
+        if (WMAX > 1) {
+            w1_rows = __ballot_sync(kFull, (mnext & 1) != 0);
+            w2_rows = __ballot_sync(kFull, (mnext & 2) != 0);
+        }
         __syncwarp();
         load_meta((blk + 1) * 32 + lane, pnext, mnext);
         uint32_t wbits[C];
@@ -371,16 +381,17 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
                     break;
                 }
             }
-            const uint32_t mbase = 1u << (sb * kSub);
-            int4 mmv[kSub];
+            const int s8 = sb * kSub;
+            const uint32_t cb = cur_rows >> s8, pb = push_rows >> s8, rb = reload_rows >> s8;
+            const uint32_t stk8 = ((push_rows | reload_rows | zero_rows) >> s8) & ((1u << kSub) - 1);
+            const uint32_t wb1 = w1_rows >> s8, wb2 = w2_rows >> s8;
+            const uint32_t sa0 = nx_ring + (uint32_t)((r0 & (kRing - 1)) * WMAX * 8);
+            uint32_t wb8[C];
 #pragma unroll
-            for (int u = 0; u < kSub; ++u) mmv[u] = my_meta[sb * kSub + u];
+            for (int c = 0; c < C; ++c) wb8[c] = 0;
             // one row of Eq. 9 for this warp's columns; STACK: the row may push or pop
             auto row = [&](const int u, const bool STACK) {
-                const int r = r0 + u;
-                const int4 mm = mmv[u];
-                const int64_t p = (int64_t)(((uint64_t)(uint32_t)mm.y << 32) | (uint32_t)mm.x);
-                const int32_t m = mm.z;
+                const int64_t p = my_p[s8 + u];
                 // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
                 // (the first warp's sv is all zero: column 0 of every row is 0)
                 int64_t bnd[WMAX];
@@ -396,54 +407,62 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int32_t *__restrict__ rowlist,
 #pragma unroll
                     for (int q = 0; q < WMAX; ++q) bnd[q] = carry[q];
                 }
+                const int w = WMAX == 1 ? 1 : 1 + (int)((wb1 >> u) & 1u) + 2 * (int)((wb2 >> u) & 1u);
                 int64_t sh[C];
-                shift_row<C, WMAX>(cur, bnd, lane0, (m & 7) + 1, sh);
-                const uint32_t mrow = mbase << u;
+                shift_row<C, WMAX>(cur, bnd, lane0, w, sh);
                 // skip row: row i+1 (a leaf) or the stack top
-                const bool from_cur = mm.w != 0;
+                const bool from_cur = (cb >> u) & 1u;
 #pragma unroll
                 for (int c = 0; c < C; ++c) {
                     const int64_t sk = from_cur ? cur[c] : top[c];
                     const int64_t t = p + sh[c];
                     const bool take = t > sk;
                     cur[c] = take ? t : sk;
-                    if (take) wbits[c] |= mrow;
+                    if (take) wb8[c] |= 1u << u;
                 }
                 // hand this row's last WMAX columns to the next warp (lane 31 only)
-                {
-                    const uint32_t sa = nx_ring + (uint32_t)(((r & (kRing - 1)) * WMAX) * 8);
 #pragma unroll
-                    for (int q = 0; q < WMAX; ++q)
-                        st_relaxed_cluster_u64_if(publish, sa + q * 8, (uint64_t)cur[C - WMAX + q] | lap);
-                }
-                // skip-row stack: push (the new row becomes the top), reload or reset the top
-                // (the flags are the same in every lane; the vote makes that visible)
-                if (STACK && __any_sync(kFull, (m & kWaveStackOps) != 0)) {
-                    const int lvl = (int)((uint32_t)m >> 16);
-                    int64_t *at = lvl < L_smem ? my_stk + (size_t)lvl * C * NT
-                                               : my_gst + (size_t)(lvl - L_smem) * CL * C * NT;
-                    if (m & kWavePush) {
+                for (int q = 0; q < WMAX; ++q)
+                    st_relaxed_cluster_u64_if(publish, sa0 + (uint32_t)((u * WMAX + q) * 8),
+                                              (uint64_t)cur[C - WMAX + q] | lap);
+                // skip-row stack (warp-uniform masks): push (the new row becomes
+                // the top), reload the new top after a pop, or reset it to the zero row
+                if (STACK && ((stk8 >> u) & 1u)) {
+                    if ((pb >> u) & 1u) {
+                        const int lvl = my_lv[s8 + u];
 #pragma unroll
-                        for (int c = 0; c < C; ++c) {
-                            top[c] = cur[c];
-                            at[(size_t)c * NT] = cur[c];
+                        for (int c = 0; c < C; ++c) top[c] = cur[c];
+                        if (lvl < L_smem) {
+#pragma unroll
+                            for (int c = 0; c < C; ++c) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < C; ++c) my_gst[(size_t)(lvl - L_smem) * CL * C * NT + (size_t)c * NT] = cur[c];
                         }
-                    } else if (m & kWaveReload) {
+                    } else if ((rb >> u) & 1u) {
+                        const int lvl = my_lv[s8 + u];
+                        if (lvl < L_smem) {
 #pragma unroll
-                        for (int c = 0; c < C; ++c) top[c] = at[(size_t)c * NT];
+                            for (int c = 0; c < C; ++c) top[c] = stk[((size_t)lvl * C + c) * NT + threadIdx.x];
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < C; ++c) top[c] = my_gst[(size_t)(lvl - L_smem) * CL * C * NT + (size_t)c * NT];
+                        }
                     } else {
 #pragma unroll
                         for (int c = 0; c < C; ++c) top[c] = 0;
                     }
                 }
             };
-            if (((stack_rows >> (sb * kSub)) & ((1u << kSub) - 1)) == 0) {
+            if (stk8 == 0) {
 #pragma unroll
                 for (int u = 0; u < kSub; ++u) row(u, false);       // no push or pop in these rows
             } else {
 #pragma unroll
                 for (int u = 0; u < kSub; ++u) row(u, true);
             }
+#pragma unroll
+            for (int c = 0; c < C; ++c) wbits[c] |= wb8[c] << s8;
             if (has_prev) {
                 // the last row of this sub-block feeds the first row of the next one
                 if (WMAX == 1) {
@@ -786,8 +805,9 @@ template <bool BYNODE>
 __global__ void __launch_bounds__(1024)
 k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
         const int32_t *__restrict__ next, const int2 *__restrict__ pspan,
-        const int32_t *__restrict__ wpre, const int32_t *__restrict__ item_active, DpWork w,
-        int prune, unsigned long long *__restrict__ rows_kept)
+        const int32_t *__restrict__ wpre, const int32_t *__restrict__ wmeta,
+        const int32_t *__restrict__ item_active, DpWork w, int prune,
+        unsigned long long *__restrict__ rows_kept)
 {
     __shared__ int sh[32];
     const int item = blockIdx.x;
@@ -842,11 +862,15 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
     int32_t *ws = w.wsuf + (size_t)item * (n + 1);
     const int kchunk = (nk + T - 1) / T;
     const int klo = min(nk, t * kchunk), khi = min(nk, klo + kchunk);
+    int64_t *rp = w.rowp + (size_t)item * n;
+    int32_t *rm = w.rowm + (size_t)item * n;
     int wsum = 0;
     for (int q = klo; q < khi; ++q) {
         const int i = rl[q];
         sk[q] = next[i] < n ? kx[next[i]] : -1;
         wsum += wpre[i];
+        rp[q] = Pp[BYNODE ? order[i] : i];     // the DP's row stream, in sweep order
+        rm[q] = wmeta[i];
     }
     int wex = block_exclusive_scan(wsum, &total, sh);     // weight of kept rows before klo
     for (int q = klo; q < khi; ++q) {
@@ -863,8 +887,8 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 size_t dp_work_bytes(int batch, int n, int words)
 {
     const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
-    return align256(B * nb * words * 4) + 4 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
-           align256(B * 4);
+    return align256(B * nb * words * 4) + 5 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
+           align256(B * 4) + align256(B * N * 8);
 }
 
 DpWork dp_work_split(void *base, int batch, int n, int words)
@@ -887,6 +911,10 @@ DpWork dp_work_split(void *base, int batch, int n, int words)
     w.skip2 = reinterpret_cast<int32_t *>(p);
     p += align256(B * N * 4);
     w.wsuf = reinterpret_cast<int32_t *>(p);
+    p += align256(B * (N + 1) * 4);
+    w.rowp = reinterpret_cast<int64_t *>(p);
+    p += align256(B * N * 8);
+    w.rowm = reinterpret_cast<int32_t *>(p);
     return w;
 }
 
@@ -1039,13 +1067,15 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
     // the pruned sweep of every item, then the DP over its kept rows
     if (by_node)
         k_prune<true><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
-                                              inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
+                                              inst->d_wpre, inst->d_wave, item_active, work, !g_tune_noprune,
+                                              rows_kept);
     else
         k_prune<false><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
-                                               inst->d_wpre, item_active, work, !g_tune_noprune, rows_kept);
+                                               inst->d_wpre, inst->d_wave, item_active, work, !g_tune_noprune,
+                                               rows_kept);
     PP_CUDA(cudaGetLastError());
     uint32_t *bits = work.bits;
-    const int32_t *rowlist = work.rowlist, *nkept = work.nkept;
+    const int32_t *nkept = work.nkept;
     if (g.wave) {
         const void *fn = wave_kernel_for(g.C, g.WMAX);
         if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
@@ -1064,11 +1094,11 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
         cfg.numAttrs = 1;
         int32_t n = inst->n;
         int32_t nblk = (n + 31) / 32;
-        const int32_t *order = by_node ? inst->d_order : nullptr;
-        const int32_t *wm = inst->d_wave;
+        const int64_t *rowp = work.rowp;
+        const int32_t *rowm = work.rowm;
         int32_t L_smem = g.L_smem, Lg = L_glob;
         int32_t *status = inst->d_status;
-        void *args[] = {&n, &nblk, (void *)&rowlist, (void *)&nkept, (void *)&profit, (void *)&order, (void *)&wm, (void *)&item_budget, &max_budget,
+        void *args[] = {&n, &nblk, (void *)&rowp, (void *)&rowm, (void *)&nkept, (void *)&item_budget, &max_budget,
                         (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status};
         PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
         return PP_OK;

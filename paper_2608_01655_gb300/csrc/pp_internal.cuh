@@ -93,6 +93,8 @@ struct DpWork {
     int32_t *skip = nullptr;       // [batch][n]
     int32_t *skip2 = nullptr;      // [batch][n]
     int32_t *wsuf = nullptr;       // [batch][n + 1]
+    int64_t *rowp = nullptr;       // [batch][n] profit of each kept row, sweep order
+    int32_t *rowm = nullptr;       // [batch][n] wave-kernel metadata of each kept row
 };
 size_t dp_work_bytes(int batch, int n, int words);
 DpWork dp_work_split(void *base, int batch, int n, int words);
