@@ -199,6 +199,75 @@ def _traffic_record():
     return None
 
 
+def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, stream):
+    """Read bandwidth of L2 and HBM (pp_probe_read), the per-row time of the
+    smallest DP launch shape (one warp per DP, 32 columns: the dependent row
+    chain with no hand-off between warps), and the B_stream model of the
+    paper's table algorithm (every row with next(i) != i+1 gathers a whole
+    skip row from memory)."""
+    sink = torch.zeros(1, dtype=torch.int64, device="cuda")
+
+    def read_gbs(nbytes, iters):
+        buf = torch.ones(nbytes // 8, dtype=torch.int64, device="cuda")
+        pp.pp_probe_read(buf, 1, sink, stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        pp.pp_probe_read(buf, iters, sink, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        del buf
+        return nbytes * iters / (e0.elapsed_time(e1) / 1000.0) / 1e9
+
+    l2_gbs = read_gbs(32 << 20, 200)          # 32 MiB: resident in L2
+    hbm_gbs = read_gbs(4 << 30, 3)            # 4 GiB: far larger than L2
+
+    # t_row_min: the plan's last DP inputs at one warp per DP and 32 columns
+    masks = np.zeros((S, n), np.uint32)
+    for m in range(inst.W):
+        masks |= res.placement[m].astype(np.uint32) << np.uint32(m)
+    masks_t = torch.from_numpy(masks.view(np.int32)).cuda()
+    workers = torch.arange(S, dtype=torch.int32, device="cuda") % inst.W
+    prof = torch.zeros((S, n), dtype=torch.int64, device="cuda")
+    pp.pp_marginals(ppi, workers, masks_t, prof)
+    kk = 32
+    pp.pp_tune_dp(1, 1, False, False)
+    try:
+        bud = torch.full((S,), kk, dtype=torch.int32, device="cuda")
+        best = torch.zeros(S, dtype=torch.int64, device="cuda")
+        bits = torch.zeros(pp.pp_dp_bits_size(ppi, S, kk) // 4, dtype=torch.int32, device="cuda")
+        ts = []
+        for it in range(4):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            pp.pp_tree_dp(ppi, prof, bud, kk, best, bits)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if it:
+                ts.append(e0.elapsed_time(e1) / 1000.0)
+        ppi.sync()
+        rows_max = int(pp.pp_dp_rows_swept(ppi, S, kk, bits).max())
+    finally:
+        pp.pp_tune_dp(0, 0, False, False)
+    t_row_min = min(ts) / rows_max
+    # B_stream: B_min plus one (k+1)-word skip-row read for every row whose
+    # skip row is not the row just computed
+    code = pp.pp_row_plan_registers(inst.parent, inst.weight)
+    frac_gather = float(np.mean(((code >> 3) & 3) != 0))
+    bstream = bmin + rows_swept * frac_gather * 8 * (k + 1)
+    rows_item = rows_swept / items
+    return {
+        "l2_read_gbs": l2_gbs, "hbm_read_gbs": hbm_gbs,
+        "roofline_extra": {
+            "bstream_bytes_per_launch": bstream, "bstream_gbs": bstream / dp_t / 1e9,
+            "bstream_frac_of_l2": bstream / dp_t / 1e9 / l2_gbs,
+            "l2_read_gbs_probe": l2_gbs, "hbm_read_gbs_probe": hbm_gbs,
+            "t_row_min_ns": 1e9 * t_row_min,
+            "t_row_min_source": "one warp per DP, 32 columns, same rows (pp_tune_dp(1, 1))",
+            "t_dp_over_rows_x_t_row_min": dp_t / (rows_item * t_row_min),
+        },
+    }
+
+
 def run_native(args):
     import torch
     world, rank, local = _dist()
@@ -293,6 +362,10 @@ def run_native(args):
                 "hbm_bmin_frac": bmin / dp_t / 1e9 / float(peaks.get("hbm_gbs", 6800.0)),
                 "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0)), "hbm_peak_kind": peak_kind}
 
+    # ---- memory-hierarchy probes and the dependent-row bound (outside the timed region)
+    probes = _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, stream)
+    roofline.update(probes.pop("roofline_extra"))
+
     # ---- end to end through the C ABI from pinned host buffers -------------
     host = {}
     for name in ("parent", "weight", "demand", "recompute", "transfer", "budget"):
@@ -357,6 +430,9 @@ def run_native(args):
                      "step_ms": [round(1000 * t, 3) for t in times]},
             "phase_ms": {"marginals": phase_sum[0] / args.steps, "tree_dp": phase_sum[1] / args.steps,
                          "traceback_accept": phase_sum[2] / args.steps},
+            "update_ms": sum(phase_sum) / (nl * args.steps),
+            "update_note": "one batched worker update (marginals + tree DP + traceback/accept) of all starts",
+            "probes": probes,
             "dp_geometry": pp.pp_dp_geometry(ppi, S, k),
         }
         print(json.dumps(line), flush=True)

@@ -328,6 +328,17 @@ pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t f
  */
 pp_status pp_default_orders(pp_instance *inst, int32_t n_starts, int32_t *orders, void *stream);
 
+/*
+ * pp_probe_read -- benchmark helper with no counterpart in the paper: reads
+ * the device buffer `buf` (`bytes` bytes, 16-byte aligned, a multiple of 16)
+ * `iters` times with 16-byte loads that bypass L1, on all SMs.  A buffer that
+ * fits in L2 gives the L2 read bandwidth that the roofline of the DP's
+ * skip-row gathers is quoted against; a buffer far larger than L2 gives the
+ * HBM read bandwidth.  `sink` (device, 8 bytes) only keeps the loads live.
+ * Asynchronous on `stream`.  Errors: PP_EINVAL, PP_ECUDA.
+ */
+pp_status pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *sink, void *stream);
+
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);
 

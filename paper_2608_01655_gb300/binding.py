@@ -65,6 +65,7 @@ _SIGS = {
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
     "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
     "pp_default_orders": [_P, _i32, _P, _P],
+    "pp_probe_read": [_P, ctypes.c_size_t, _i32, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -290,3 +291,9 @@ def pp_default_orders(inst: Instance, n_starts: int, stream=None) -> np.ndarray:
     out = np.zeros((int(n_starts), inst.W), np.int32)
     _check(_lib.pp_default_orders(inst.handle, int(n_starts), _host(out), _stream(stream)))
     return out
+
+
+def pp_probe_read(buf, iters: int, sink, stream=None):
+    """Read the CUDA tensor `buf` `iters` times (bandwidth probe); sink: 1-element int64 CUDA tensor."""
+    _check(_lib.pp_probe_read(_dev(buf), int(buf.numel() * buf.element_size()), int(iters), _dev(sink),
+                              _stream(stream)))
