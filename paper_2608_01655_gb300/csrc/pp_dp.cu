@@ -809,6 +809,9 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         const int32_t *__restrict__ item_active, DpWork w, int prune,
         unsigned long long *__restrict__ rows_kept)
 {
+    // every pass walks tiles of T*V consecutive elements, V per thread, with one
+    // block scan per tile and a carry between tiles (all threads run every tile)
+    constexpr int V = 4;
     __shared__ int sh[32];
     const int item = blockIdx.x;
     if (item_active && !item_active[item]) return;
@@ -816,70 +819,114 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
     int32_t *cnt = w.cnt + (size_t)item * (n + 1);
     int32_t *rl = w.rowlist + (size_t)item * n;
     int32_t *kx = w.kidx + (size_t)item * n;
-    const int T = blockDim.x, t = threadIdx.x;
-    const int chunk = (n + T - 1) / T;
-    const int lo = min(n, t * chunk), hi = min(n, lo + chunk);
-    int total = 0;
+    const int T = blockDim.x, t = threadIdx.x, tile = T * V;
+    auto pval = [&](int i) { return Pp[BYNODE ? order[i] : i]; };
+
     // prefix counts of positive profits, preorder
-    int c = 0;
-    for (int i = lo; i < hi; ++i) c += Pp[BYNODE ? order[i] : i] > 0;
-    int ex = block_exclusive_scan(c, &total, sh);
-    for (int i = lo; i < hi; ++i) {
-        cnt[i] = ex;
-        ex += Pp[BYNODE ? order[i] : i] > 0;
+    int carry = 0;
+    for (int base = 0; base < n; base += tile) {
+        int f[V], c = 0, total;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int i = base + t * V + v;
+            f[v] = i < n && pval(i) > 0;
+            c += f[v];
+        }
+        int ex = block_exclusive_scan(c, &total, sh) + carry;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int i = base + t * V + v;
+            if (i < n) {
+                cnt[i] = ex;
+                ex += f[v];
+            }
+        }
+        carry += total;
     }
-    if (t == 0) cnt[n] = total;
+    if (t == 0) cnt[n] = carry;
     __syncthreads();
-    // kept rows in sweep order r = n - 1 - i; the flag goes to kx[i] first
-    // (0 kept, -1 dropped) and is replaced by the kept index below
-    int kc = 0;
-    for (int r = lo; r < hi; ++r) {
-        const int i = n - 1 - r;
-        bool kp = true;
-        if (prune) {
-            const int2 sp = pspan[i];
-            kp = sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0;
+
+    // kept rows in sweep order r = n - 1 - i, their kept index, their total weight
+    int kcarry = 0, wmine = 0;
+    for (int base = 0; base < n; base += tile) {
+        bool kp[V];
+        int kc = 0, total;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int r = base + t * V + v;
+            kp[v] = false;
+            if (r < n) {
+                kp[v] = true;
+                if (prune) {
+                    const int2 sp = pspan[n - 1 - r];
+                    kp[v] = sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0;
+                }
+            }
+            kc += kp[v];
         }
-        kx[i] = kp ? 0 : -1;
-        kc += kp;
-    }
-    int kex = block_exclusive_scan(kc, &total, sh);
-    for (int r = lo; r < hi; ++r) {
-        const int i = n - 1 - r;
-        if (kx[i] == 0) {
-            rl[kex] = i;
-            kx[i] = kex++;
+        int ex = block_exclusive_scan(kc, &total, sh) + kcarry;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int r = base + t * V + v;
+            if (r < n) {
+                const int i = n - 1 - r;
+                if (kp[v]) {
+                    rl[ex] = i;
+                    kx[i] = ex++;
+                    wmine += wpre[i];
+                } else {
+                    kx[i] = -1;
+                }
+            }
         }
+        kcarry += total;
     }
-    const int nk = total;
+    const int nk = kcarry;
+    int wtot;
+    block_exclusive_scan(wmine, &wtot, sh);                // weight of all kept rows
     if (t == 0) {
         w.nkept[item] = nk;
         if (rows_kept) atomicAdd(rows_kept, (unsigned long long)nk);
     }
     __syncthreads();
-    // traceback tables over kept rows: skip targets and suffix weights
+
+    // per kept row: skip target, the DP's row stream (profit, metadata) and
+    // the suffix weights of the traceback
     int32_t *sk = w.skip + (size_t)item * n, *sk2 = w.skip2 + (size_t)item * n;
     int32_t *ws = w.wsuf + (size_t)item * (n + 1);
-    const int kchunk = (nk + T - 1) / T;
-    const int klo = min(nk, t * kchunk), khi = min(nk, klo + kchunk);
     int64_t *rp = w.rowp + (size_t)item * n;
     int32_t *rm = w.rowm + (size_t)item * n;
-    int wsum = 0;
-    for (int q = klo; q < khi; ++q) {
-        const int i = rl[q];
-        sk[q] = next[i] < n ? kx[next[i]] : -1;
-        wsum += wpre[i];
-        rp[q] = Pp[BYNODE ? order[i] : i];     // the DP's row stream, in sweep order
-        rm[q] = wmeta[i];
-    }
-    int wex = block_exclusive_scan(wsum, &total, sh);     // weight of kept rows before klo
-    for (int q = klo; q < khi; ++q) {
-        ws[q] = total - wex;                               // weight of kept rows q..nk-1
-        wex += wpre[rl[q]];
+    int wcarry = 0;
+    for (int base = 0; base < nk; base += tile) {
+        int wq[V], wl = 0, total;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int q = base + t * V + v;
+            wq[v] = 0;
+            if (q < nk) {
+                const int i = rl[q];
+                const int nx = next[i];
+                sk[q] = nx < n ? kx[nx] : -1;
+                wq[v] = wpre[i];
+                rp[q] = pval(i);
+                rm[q] = wmeta[i];
+            }
+            wl += wq[v];
+        }
+        int ex = block_exclusive_scan(wl, &total, sh) + wcarry;   // weight of kept rows before q
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int q = base + t * V + v;
+            if (q < nk) {
+                ws[q] = wtot - ex;                                 // weight of kept rows q..nk-1
+                ex += wq[v];
+            }
+        }
+        wcarry += total;
     }
     if (t == 0) ws[nk] = 0;
     __syncthreads();
-    for (int q = klo; q < khi; ++q) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
+    for (int q = t; q < nk; q += T) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
 }
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
