@@ -60,7 +60,8 @@ def _load():
             "or_rooted_dp": (i64, [i32, P, P, P, i32, P, ctypes.c_int]),
             "or_standalone": (ctypes.c_int, [P, P]),
             "or_default_orders": (ctypes.c_int, [P, i32, P]),
-            "or_plan": (i32, [P, i32, P, i32, i32, P, P, P, P, P, P]),
+            "or_plan": (i32, [P, i32, P, i32, i32, P, P, P, P, P, P, ctypes.c_int, P]),
+            "or_safeguards": (ctypes.c_int, [P, P, P]),
             "or_worker_update": (i64, [P, i32, P, P, P]),
         }
         for name, (res, args) in sig.items():
@@ -181,10 +182,28 @@ class PlanResult:
     per_start_sweeps: np.ndarray
     per_start_accepted: np.ndarray
     cells: int
+    safeguard_objective: np.ndarray | None = None   # [3] when the safeguards took part
 
 
-def plan(prob: Problem, S: int, R: int, orders=None, threads: int | None = None) -> PlanResult:
-    """Algorithm 1 over S starts and at most R refinement sweeps."""
+def safeguards(prob: Problem):
+    """Independent, Popularity and LocalDedup placements (requester-side only).
+
+    Returns (placement [3][W][n] uint8, objective [3] int64)."""
+    pl = np.zeros((3, prob.W, max(prob.n, 1)), np.uint8)
+    obj = np.zeros(3, np.int64)
+    r = _load().or_safeguards(prob.ref, _ptr(pl), _ptr(obj))
+    if r == -2:
+        raise ValueError("safeguard candidates are defined for the requester-side objective only")
+    if r != 0:
+        raise ValueError("parent array is not a forest")
+    return pl[:, :, :prob.n].copy(), obj
+
+
+def plan(prob: Problem, S: int, R: int, orders=None, threads: int | None = None,
+         safeguards: bool = True) -> PlanResult:
+    """Algorithm 1 over S starts and at most R refinement sweeps; with the
+    requester-side objective the safeguard candidates join as indices S..S+2
+    unless safeguards=False."""
     if threads is None:
         threads = min(S, os.cpu_count() or 1)
     pl = np.zeros((prob.W, max(prob.n, 1)), np.uint8)
@@ -198,11 +217,15 @@ def plan(prob: Problem, S: int, R: int, orders=None, threads: int | None = None)
         orders = _c(orders, np.int32)
         assert orders.shape == (S, prob.W)
         op = _ptr(orders)
+    sg = np.zeros(3, np.int64)
     best = _load().or_plan(prob.ref, int(S), op, int(R), int(threads), _ptr(pl), ctypes.byref(obj),
-                           _ptr(per), _ptr(sw), _ptr(acc), ctypes.byref(cells))
+                           _ptr(per), _ptr(sw), _ptr(acc), ctypes.byref(cells), int(bool(safeguards)),
+                           _ptr(sg))
     if best < 0:
         raise ValueError("parent array is not a forest")
-    return PlanResult(pl[:, :prob.n].copy(), int(obj.value), int(best), per, sw, acc, int(cells.value))
+    used = bool(safeguards) and prob.mode == 0
+    return PlanResult(pl[:, :prob.n].copy(), int(obj.value), int(best), per, sw, acc, int(cells.value),
+                      sg if used else None)
 
 
 def worker_update(prob: Problem, h: int, placement):

@@ -29,8 +29,10 @@
  *   or_rooted_dp       Eq. 9, Theorem 1, Algorithm 1 procedure RootedDP
  *   or_standalone      standalone score (Section IV-C, Algorithm 1)
  *   or_default_orders  start orders (Section IV-C); permutations by SplitMix64
+ *   or_safeguards      Algorithm 1's safeguard candidates (requester-side):
+ *                      Independent, Popularity, LocalDedup (Sections IV-C, V-A)
  *   or_plan            Algorithm 1 procedure PrefixPlace (greedy, refinement,
- *                      starts; safeguard candidates are not included)
+ *                      starts, and the safeguard candidates when asked for)
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -432,6 +434,51 @@ static void run_start(or_start *st)
     free(p); free(Tnew); free(Told);
 }
 
+/* ------------------------------------------------------------------------ */
+/* Safeguard candidates (Algorithm 1, requester-side objective only; the    */
+/* comparators of Section V-A).  Every worker's target is RootedDP(p, k_m)  */
+/* with                                                                      */
+/*   Independent  p(b) = Lambda_m(b) w_m(b): local demand weighted by       */
+/*                recomputation cost, cross-worker reuse ignored;           */
+/*   Popularity   p(b) = Lambda_m(b): local demand alone;                   */
+/*   LocalDedup   workers in index order; a chunk that an earlier worker     */
+/*                already holds is worth only the local value a_m(b) of     */
+/*                Eq. 2, any other chunk Lambda_m(b) w_m(b) -- the worker's  */
+/*                own saving from the first copy, not the requester-wide     */
+/*                Delta(b) of Eq. 3.                                         */
+/* placement: [3][W][n] out (Independent, Popularity, LocalDedup);           */
+/* objective: [3] out, Eq. 4.  Returns 0; -1 if parent[] is not a forest;    */
+/* -2 in the source-dependent mode (Algorithm 1 adds them only for the       */
+/* requester-side objective).                                                */
+/* ------------------------------------------------------------------------ */
+int or_safeguards(const or_inst *I, uint8_t *placement, int64_t *objective)
+{
+    if (I->mode != 0) return -2;
+    int32_t n = I->n, W = I->W;
+    int32_t *order = malloc(sizeof(int32_t) * ((size_t)n + 1));
+    int32_t *next = malloc(sizeof(int32_t) * ((size_t)n + 1));
+    if (or_preorder(n, I->parent, order, next) != 0) { free(order); free(next); return -1; }
+    int64_t *p = malloc(sizeof(int64_t) * ((size_t)n + 1));
+    uint8_t *held = calloc((size_t)n + 1, 1);     /* LocalDedup: held by an earlier worker */
+    memset(placement, 0, (size_t)3 * W * n);
+    for (int32_t c = 0; c < 3; ++c) {
+        uint8_t *X = placement + (size_t)c * W * n;
+        for (int32_t m = 0; m < W; ++m) {
+            for (int32_t b = 0; b < n; ++b) {
+                if (c == 0) p[b] = LAM(I, m, b) * WCOST(I, m, b);
+                else if (c == 1) p[b] = LAM(I, m, b);
+                else p[b] = held[b] ? eq2_local_value(I, m, b) : LAM(I, m, b) * WCOST(I, m, b);
+            }
+            or_rooted_dp_pre(n, order, next, I->weight, p, I->budget[m], X + (size_t)m * n, -1);
+            if (c == 2)
+                for (int32_t b = 0; b < n; ++b) held[b] |= X[(size_t)m * n + b];
+        }
+        objective[c] = or_objective(I, X);
+    }
+    free(order); free(next); free(p); free(held);
+    return 0;
+}
+
 typedef struct {
     or_start *starts;
     int32_t S;
@@ -452,12 +499,17 @@ static void *pool_worker(void *arg)
 }
 
 /* orders: [S][W] or NULL (then or_default_orders).  placement: [W][n] out, */
-/* the best start's targets (highest objective, ties to the lowest start).  */
-/* per_start_obj / sweeps / accepted: [S] out or NULL.  Returns the best    */
-/* start index, or -1 on an invalid tree.                                    */
+/* the best candidate's targets (highest objective, ties to the lowest      */
+/* index).  With safeguards != 0 and the requester-side objective, the      */
+/* Independent, Popularity and LocalDedup placements join the candidates as */
+/* indices S, S+1, S+2 (Algorithm 1), and safeguard_obj [3] receives their  */
+/* objectives (else it is left alone).  per_start_obj / sweeps / accepted:  */
+/* [S] out or NULL.  Returns the best candidate index, or -1 on an invalid  */
+/* tree.                                                                     */
 int32_t or_plan(const or_inst *I, int32_t S, const int32_t *orders, int32_t R, int32_t n_threads,
                 uint8_t *placement, int64_t *objective, int64_t *per_start_obj,
-                int32_t *per_start_sweeps, int32_t *per_start_accepted, int64_t *cells_out)
+                int32_t *per_start_sweeps, int32_t *per_start_accepted, int64_t *cells_out,
+                int safeguards, int64_t *safeguard_obj)
 {
     int32_t n = I->n, W = I->W;
     int32_t *order = malloc(sizeof(int32_t) * ((size_t)n + 1));
@@ -490,9 +542,25 @@ int32_t or_plan(const or_inst *I, int32_t S, const int32_t *orders, int32_t R, i
     }
     if (!orders && S > 1)                      /* the standalone-score DPs of the default orders */
         for (int32_t m = 0; m < W; ++m) cells += (int64_t)n * I->budget[m];
-    if (cells_out) *cells_out = cells;
     memcpy(placement, st[best].T, (size_t)W * n);
     *objective = st[best].objective;
+    if (safeguards && I->mode == 0) {
+        uint8_t *X = malloc((size_t)3 * W * n + 1);
+        int64_t so[3];
+        or_safeguards(I, X, so);
+        for (int32_t c = 0; c < 3; ++c) {
+            if (safeguard_obj) safeguard_obj[c] = so[c];
+            if (so[c] > *objective) {
+                *objective = so[c];
+                best = S + c;
+                memcpy(placement, X + (size_t)c * W * n, (size_t)W * n);
+            }
+        }
+        for (int32_t c = 0; c < 3; ++c)        /* one DP per worker and candidate */
+            for (int32_t m = 0; m < W; ++m) cells += (int64_t)n * I->budget[m];
+        free(X);
+    }
+    if (cells_out) *cells_out = cells;
     free(th); free(st); free(T); free(order); free(next); free(ord);
     return best;
 }

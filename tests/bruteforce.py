@@ -106,3 +106,33 @@ def is_parent_closed(parent, chosen) -> bool:
     ch = np.asarray(chosen, bool)
     has_p = parent >= 0
     return bool(np.all(~ch[has_p] | ch[parent[has_p]]))
+
+
+def requester_saving(inst, placement, m) -> int:
+    """Requester m's own saving over all-recompute under the Section III-A rule
+    (local copy 0, otherwise the cheapest of w_m and a fetch from any holder)."""
+    pl = np.asarray(placement, bool)
+    total = 0
+    for b in range(inst.n):
+        w = int(inst.recompute[m, b])
+        holders = [h for h in range(inst.W) if pl[h, b]]
+        if pl[m, b]:
+            cost = 0
+        elif holders:
+            fetch = int(inst.transfer[m, b]) if inst.mode == 0 else min(int(inst.transfer[h, m, b]) for h in holders)
+            cost = min(w, fetch)
+        else:
+            cost = w
+        total += int(inst.demand[m, b]) * (w - cost)
+    return total
+
+
+def best_set_by(parent, weight, k, value):
+    """Parent-closed set of weight <= k maximising value(mask); ties to the
+    lexicographically smallest preorder indicator (the DP's rule)."""
+    sets = parent_closed_masks(parent, weight, k)
+    vals = [value(s) for s in sets]
+    best = max(vals)
+    order = preorder_positions(parent)
+    cand = [s for s, v in zip(sets, vals) if v == best]
+    return min(cand, key=lambda s: tuple(int(s[v]) for v in order)).astype(np.uint8)

@@ -315,6 +315,93 @@ def test_generator_constants_match_paper_arithmetic():
     assert wl.ALPHA_US_PER_TOKEN[2] == 8 * wl.ALPHA_US_PER_TOKEN[0]
 
 
+# ------------------------------------------------- safeguard candidates ---
+def test_safeguards_match_their_definitions(oracle_lib):
+    """Algorithm 1's requester-side safeguards (Section IV-C, comparators of
+    Section V-A), each worker's set found by enumeration from the Section III-A
+    saving rule rather than from a profit formula:
+      Independent  maximises requester m's own saving with no other copy;
+      Popularity   maximises requester m's local hits (its demand);
+      LocalDedup   in index order, maximises requester m's own saving given
+                   the sets of the earlier workers (later ones empty)."""
+    rng = np.random.default_rng(71)
+    for trial in range(25):
+        W = int(rng.integers(1, 4))
+        inst = wl.random_small(rng, int(rng.integers(1, 9)), W, 0, k_max=4, w_max=2)
+        pl, obj = oracle_lib.safeguards(_prob(oracle_lib, inst))
+        n = inst.n
+        hits = wl.Instance(**{**inst.__dict__, "recompute": np.ones_like(inst.recompute),
+                              "transfer": np.full_like(inst.transfer, 2)})
+        dedup = np.zeros((W, n), np.uint8)
+        for m in range(W):
+            def alone(s, src=inst):
+                x = np.zeros((W, n), np.uint8)
+                x[m] = s
+                return bf.requester_saving(src, x, m)
+
+            def after_earlier(s):
+                x = dedup.copy()
+                x[m] = s
+                return bf.requester_saving(inst, x, m)
+            k = int(inst.budget[m])
+            np.testing.assert_array_equal(pl[0, m], bf.best_set_by(inst.parent, inst.weight, k, alone))
+            np.testing.assert_array_equal(pl[1, m], bf.best_set_by(inst.parent, inst.weight, k,
+                                                                   lambda s: alone(s, hits)))
+            dedup[m] = bf.best_set_by(inst.parent, inst.weight, k, after_earlier)
+        np.testing.assert_array_equal(pl[2], dedup)
+        for c in range(3):
+            assert obj[c] == bf.materialisation_saving(inst, pl[c])
+
+
+def test_safeguards_special_cases(oracle_lib):
+    """With one worker Independent and LocalDedup coincide (nothing earlier to
+    discount); when every fetch costs at least the recomputation the
+    discounted value min{w, f} equals w, so LocalDedup is Independent again;
+    with unit recomputation cost Independent is Popularity."""
+    rng = np.random.default_rng(72)
+    for trial in range(20):
+        inst = wl.random_small(rng, int(rng.integers(1, 30)), 1, 0, k_max=10, w_max=3)
+        pl, _ = oracle_lib.safeguards(_prob(oracle_lib, inst))
+        np.testing.assert_array_equal(pl[0], pl[2])
+        W = int(rng.integers(2, 5))
+        inst = wl.random_small(rng, int(rng.integers(1, 30)), W, 0, k_max=10, w_max=3)
+        slow = wl.Instance(**{**inst.__dict__, "transfer": inst.recompute + inst.transfer})
+        pl, _ = oracle_lib.safeguards(_prob(oracle_lib, slow))
+        np.testing.assert_array_equal(pl[0], pl[2])
+        ones = wl.Instance(**{**inst.__dict__, "recompute": np.ones_like(inst.recompute)})
+        pl, _ = oracle_lib.safeguards(_prob(oracle_lib, ones))
+        np.testing.assert_array_equal(pl[0], pl[1])
+
+
+def test_plan_never_worse_than_safeguards(oracle_lib):
+    """Section IV-C: the returned placement is never worse than Independent,
+    Popularity or LocalDedup under the same objective; a safeguard that beats
+    every start is returned as candidate S + c; the source-dependent objective
+    has no safeguards."""
+    rng = np.random.default_rng(73)
+    won = 0
+    for trial in range(30):
+        inst = wl.random_small(rng, int(rng.integers(2, 25)), int(rng.integers(2, 5)), 0, k_max=6, w_max=2)
+        prob = _prob(oracle_lib, inst)
+        S = int(rng.integers(1, 4))
+        with_sg = oracle_lib.plan(prob, S, 3, threads=1)
+        without = oracle_lib.plan(prob, S, 3, threads=1, safeguards=False)
+        _, obj = oracle_lib.safeguards(prob)
+        np.testing.assert_array_equal(with_sg.safeguard_objective, obj)
+        assert with_sg.objective == max(without.objective, int(obj.max()))
+        assert with_sg.objective == bf.materialisation_saving(inst, with_sg.placement)
+        if with_sg.best_start >= S:
+            won += 1
+            assert obj[with_sg.best_start - S] == with_sg.objective > without.objective
+        else:
+            assert with_sg.best_start == without.best_start
+    src = wl.random_small(rng, 10, 3, 1)
+    r = oracle_lib.plan(_prob(oracle_lib, src), 2, 2, threads=1)
+    assert r.safeguard_objective is None and r.best_start < 2
+    with pytest.raises(ValueError):
+        oracle_lib.safeguards(_prob(oracle_lib, src))
+
+
 def test_refinement_accepts_only_strict_improvements(oracle_lib):
     """Section IV-C: only strictly improving replacements are accepted, so a
     greedy result that is already coordinate-wise optimal ends after exactly
