@@ -62,7 +62,8 @@ typedef struct {
     int32_t *per_start_sweeps;     /* [n_starts] host, out: refinement sweeps run */
     int32_t *per_start_accepted;   /* [n_starts] host, out: accepted refinement updates */
     int32_t *orders_used;          /* [n_starts][W] host, out: the start orders */
-    int32_t best_start;            /* out: index of the returned candidate */
+    int32_t best_start;            /* out: index of the returned candidate (>= n_starts:
+                                      safeguard best_start - n_starts) */
     int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded) */
     int64_t dp_cells;              /* out: sum over executed DPs of n * k_h (Eq. 9 cells) */
     int32_t kernel_launches;       /* out: kernels launched by this call */
@@ -72,6 +73,9 @@ typedef struct {
                                       tree-DP (with its row pruning) and traceback launches,
                                       summed over the plan */
     int32_t dp_launches;           /* out: batched tree-DP launches (one per plan step) */
+    int32_t no_safeguards;         /* in: nonzero = leave out the safeguard candidates */
+    int64_t safeguard_objective[3];/* out: Independent, Popularity, LocalDedup objectives
+                                      (requester-side only; else 0) */
 } pp_plan_stats;
 
 /*
@@ -263,10 +267,12 @@ pp_status pp_objective(pp_instance *inst, int32_t batch, const uint8_t *chosen, 
                        void *stream);
 
 /*
- * pp_plan_run -- Algorithm 1 (procedure PrefixPlace) without the
- * requester-side safeguard candidates: for each start order, one
- * WorkerGreedy pass (Theorem 3), then at most max_rounds refinement sweeps;
- * a sweep with no accepted update ends that start.  Starts run batched.
+ * pp_plan_run -- Algorithm 1 (procedure PrefixPlace): for each start order,
+ * one WorkerGreedy pass (Theorem 3), then at most max_rounds refinement
+ * sweeps; a sweep with no accepted update ends that start.  Starts run
+ * batched.  With the requester-side objective the Independent, Popularity
+ * and LocalDedup placements (pp_safeguards) join the candidates as indices
+ * S, S+1, S+2 unless stats->no_safeguards is set.
  *   n_starts      S >= 1
  *   orders        host [S][W] permutations of 0..W-1, or NULL for the default:
  *                 S == 1 the identity; otherwise start 0 = standalone-score
@@ -275,7 +281,7 @@ pp_status pp_objective(pp_instance *inst, int32_t batch, const uint8_t *chosen, 
  *                 SplitMix64 seeded with s (j = next() mod (i + 1), i = W-1..1)
  *   max_rounds    R >= 0 refinement sweeps
  *   placement     host [W][n] out: the best candidate (highest objective,
- *                 ties to the lowest start), 1 = resident
+ *                 ties to the lowest candidate index), 1 = resident
  *   objective     host out: its objective (Eq. 4 or Eq. 6)
  *   stats         optional (NULL) extra outputs
  * Synchronous: returns after the result is on the host.  Errors: PP_EINVAL,
@@ -338,6 +344,21 @@ pp_status pp_default_orders(pp_instance *inst, int32_t n_starts, int32_t *orders
  * Asynchronous on `stream`.  Errors: PP_EINVAL, PP_ECUDA.
  */
 pp_status pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *sink, void *stream);
+
+/*
+ * pp_safeguards -- the safeguard candidates that Algorithm 1 adds for the
+ * requester-side objective (Section IV-C; the comparators of Section V-A):
+ * every worker's target is the exact DP of Eq. 9 on
+ *   [0] Independent  Lambda_m(b) w_m(b)   (the worker alone)
+ *   [1] Popularity   Lambda_m(b)          (local demand alone)
+ *   [2] LocalDedup   workers in index order; a_m(b) (Eq. 2) for a chunk an
+ *                    earlier worker holds, else Lambda_m(b) w_m(b)
+ *   placement   host [3][W][n] out, by node id
+ *   objective   host [3] out, Eq. 4
+ * Synchronous on `stream`.  Errors: PP_EINVAL (source-dependent instance,
+ * null argument, another current device), PP_ENOMEM, PP_ECUDA.
+ */
+pp_status pp_safeguards(pp_instance *inst, uint8_t *placement, int64_t *objective, void *stream);
 
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);

@@ -44,7 +44,8 @@ class PlanStats(ctypes.Structure):
     _fields_ = [("per_start_objective", _P), ("per_start_sweeps", _P), ("per_start_accepted", _P),
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
                 ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
-                ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32)]
+                ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32), ("no_safeguards", _i32),
+                ("safeguard_objective", ctypes.c_int64 * 3)]
 
 
 _SIGS = {
@@ -66,6 +67,7 @@ _SIGS = {
     "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
     "pp_default_orders": [_P, _i32, _P, _P],
     "pp_probe_read": [_P, ctypes.c_size_t, _i32, _P, _P],
+    "pp_safeguards": [_P, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -239,10 +241,11 @@ class PlanResult:
     phase_ms: tuple = ()
     dp_rows_swept: int = 0
     dp_launches: int = 0
+    safeguard_objective: tuple = ()     # Independent, Popularity, LocalDedup (requester-side)
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
-                time_phases: bool = False) -> PlanResult:
+                time_phases: bool = False, safeguards: bool = True) -> PlanResult:
     S, W, n = int(n_starts), inst.W, inst.n
     placement = np.zeros((W, max(n, 1)), np.uint8)
     obj = _i64(0)
@@ -252,6 +255,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     used = np.zeros((S, W), np.int32)
     st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0, 0,
                    int(bool(time_phases)))
+    st.no_safeguards = int(not safeguards)
     op = None
     if orders is not None:
         orders = _np(orders, np.int32)
@@ -263,7 +267,8 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     return PlanResult(placement[:, :n].copy(), int(obj.value), int(st.best_start), per, sw, acc, used,
                       int(st.dp_count), int(st.dp_cells), int(st.kernel_launches),
                       tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept),
-                      int(st.dp_launches))
+                      int(st.dp_launches),
+                      tuple(int(x) for x in st.safeguard_objective) if safeguards and inst.mode == 0 else ())
 
 
 def pp_test_inject(kind: int, value: int):
@@ -297,3 +302,11 @@ def pp_probe_read(buf, iters: int, sink, stream=None):
     """Read the CUDA tensor `buf` `iters` times (bandwidth probe); sink: 1-element int64 CUDA tensor."""
     _check(_lib.pp_probe_read(_dev(buf), int(buf.numel() * buf.element_size()), int(iters), _dev(sink),
                               _stream(stream)))
+
+
+def pp_safeguards(inst: Instance, stream=None):
+    """Independent, Popularity, LocalDedup placements [3][W][n] uint8 and objectives [3] int64."""
+    pl = np.zeros((3, inst.W, max(inst.n, 1)), np.uint8)
+    obj = np.zeros(3, np.int64)
+    _check(_lib.pp_safeguards(inst.handle, _host(pl), _host(obj), _stream(stream)))
+    return pl[:, :, :inst.n].copy(), obj

@@ -163,7 +163,8 @@ __global__ void k_gain_requester(int32_t n, int32_t W, const int32_t *__restrict
                                  const int64_t *__restrict__ demand,
                                  const int64_t *__restrict__ recompute,
                                  const int64_t *__restrict__ transfer, int64_t *__restrict__ a,
-                                 int64_t *__restrict__ delta)
+                                 int64_t *__restrict__ delta, int64_t *__restrict__ own,
+                                 int64_t *__restrict__ pop)
 {
     for (int32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
         int32_t b = order[i];
@@ -172,6 +173,8 @@ __global__ void k_gain_requester(int32_t n, int32_t W, const int32_t *__restrict
             size_t o = (size_t)m * n + b;
             int64_t lam = demand[o], w = recompute[o], f = transfer[o];
             a[(size_t)m * n + i] = lam * (w < f ? w : f);
+            own[(size_t)m * n + i] = lam * (w > f ? w - f : 0);
+            pop[(size_t)m * n + i] = lam;
             d += lam * (w > f ? w - f : 0);
         }
         delta[i] = d;
@@ -219,11 +222,14 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     cudaFree(inst->d_budget);
     cudaFree(inst->d_a);
     cudaFree(inst->d_delta);
+    cudaFree(inst->d_own);
+    cudaFree(inst->d_pop);
     cudaFree(inst->d_g);
     cudaFree(inst->d_status);
     free_scratch(inst->stack);
     free_scratch(inst->plan);
     free_scratch(inst->plan_bits);
+    free_scratch(inst->sg);
     cudaSetDevice(cur);
     delete inst;
     return PP_OK;
@@ -320,9 +326,11 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if (mode == PP_TRANSFER_REQUESTER) {
         e = cudaMalloc(&inst->d_a, sizeof(int64_t) * (Wn ? Wn : 1));
         if (e == cudaSuccess) e = cudaMalloc(&inst->d_delta, sizeof(int64_t) * (n ? n : 1));
+        if (e == cudaSuccess) e = cudaMalloc(&inst->d_own, sizeof(int64_t) * (Wn ? Wn : 1));
+        if (e == cudaSuccess) e = cudaMalloc(&inst->d_pop, sizeof(int64_t) * (Wn ? Wn : 1));
         if (e == cudaSuccess && n > 0)
             k_gain_requester<<<blocks, 256, 0, st>>>(n, W, inst->d_order, d_dem, d_rec, d_tr,
-                                                     inst->d_a, inst->d_delta);
+                                                     inst->d_a, inst->d_delta, inst->d_own, inst->d_pop);
     } else {
         e = cudaMalloc(&inst->d_g, sizeof(int64_t) * (tn ? tn : 1));
         if (e == cudaSuccess && n > 0) {

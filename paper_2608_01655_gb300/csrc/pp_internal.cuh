@@ -129,11 +129,14 @@ struct pp_instance {
     int32_t *d_budget = nullptr;        // [W]
     int64_t *d_a = nullptr;             // mode 0: [W][n] a_m(b)       (Eq. 2)
     int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)
+    int64_t *d_own = nullptr;           // mode 0: [W][n] Lambda_m(b) [w_m(b) - f_m(b)]_+ (own first-copy gain)
+    int64_t *d_pop = nullptr;           // mode 0: [W][n] Lambda_m(b)
     int64_t *d_g = nullptr;             // mode 1: [W][W][n] Lambda_m(b) q_{m<-h}(b) at [h][m][i] (Eq. 5)
     int32_t *d_status = nullptr;        // device status word
     pp::Scratch stack;                  // skip-row stack spill of pp_tree_dp
     pp::Scratch plan;                   // pp_plan_run working set
     pp::Scratch plan_bits;              // pp_plan_run decision bits
+    pp::Scratch sg;                     // safeguard candidates' working set
 };
 
 namespace pp {
@@ -185,5 +188,12 @@ struct AcceptArgs {
 pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, const DpGeom &g,
                            const int32_t *item_budget, uint8_t *chosen, const AcceptArgs *acc,
                            cudaStream_t st);
+
+// Safeguard candidates (requester-side): Independent, Popularity, LocalDedup
+// holder masks [3][n] in preorder (device, in inst->sg, valid until the next
+// call) and their objectives (host [3]).  Adds its kernel launches and DP
+// cells to the counters.
+pp_status safeguards_impl(pp_instance *inst, cudaStream_t st, const uint32_t **masks, int64_t *obj,
+                          int *launches, int64_t *cells, int *dp_launches);
 
 }  // namespace pp

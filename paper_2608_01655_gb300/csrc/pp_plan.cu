@@ -261,9 +261,24 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
     int32_t bs = 0;
     for (int32_t x = 1; x < S; ++x)
         if (obj[x] > obj[bs]) bs = x;
+    int64_t best_obj = obj[bs];
+    const uint32_t *best_mask = pb.mask + (size_t)bs * n;
+    // requester-side safeguard candidates S, S+1, S+2 (ties stay with the lower index)
+    int64_t so[3] = {0, 0, 0};
+    if (inst->mode == PP_TRANSFER_REQUESTER && !(stats && stats->no_safeguards)) {
+        const uint32_t *sgm = nullptr;
+        if ((s = safeguards_impl(inst, st, &sgm, so, &launches, &cells, &dp_launches))) return s;
+        dp_count += 3 * W;
+        for (int c = 0; c < 3; ++c)
+            if (so[c] > best_obj) {
+                best_obj = so[c];
+                bs = S + c;
+                best_mask = sgm + (size_t)c * n;
+            }
+    }
     std::vector<uint32_t> mk(std::max(n, 1));
     if (n > 0) {
-        PP_CUDA(cudaMemcpyAsync(mk.data(), pb.mask + (size_t)bs * n, 4 * (size_t)n, cudaMemcpyDeviceToHost, st));
+        PP_CUDA(cudaMemcpyAsync(mk.data(), best_mask, 4 * (size_t)n, cudaMemcpyDeviceToHost, st));
         PP_CUDA(cudaStreamSynchronize(st));
     }
     std::memset(placement, 0, (size_t)W * n);
@@ -276,7 +291,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
             placement[(size_t)h * n + b] = 1;
         }
     }
-    *objective = obj[bs];
+    *objective = best_obj;
     if (stats) {
         if (stats->per_start_objective) std::copy(obj.begin(), obj.end(), stats->per_start_objective);
         if (stats->per_start_sweeps) std::copy(sw.begin(), sw.end(), stats->per_start_sweeps);
@@ -287,6 +302,7 @@ static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, 
         stats->kernel_launches = launches;
         stats->dp_rows_swept = (int64_t)rows_swept;
         stats->dp_launches = dp_launches;
+        for (int c = 0; c < 3; ++c) stats->safeguard_objective[c] = so[c];
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
         for (size_t x = 0; x + 3 < ev.v.size(); x += 4) {
             float a = 0.f, b = 0.f, c = 0.f;

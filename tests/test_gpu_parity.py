@@ -144,6 +144,52 @@ def _compare_plans(g, o):
     np.testing.assert_array_equal(g.per_start_objective, o.per_start_objective)
     np.testing.assert_array_equal(g.per_start_sweeps, o.per_start_sweeps)
     np.testing.assert_array_equal(g.per_start_accepted, o.per_start_accepted)
+    if o.safeguard_objective is None:
+        assert g.safeguard_objective == ()
+    else:
+        assert list(g.safeguard_objective) == o.safeguard_objective.tolist()
+
+
+def test_safeguards_match_oracle(pp, oracle_lib):
+    """Independent, Popularity and LocalDedup (Algorithm 1, requester-side):
+    every worker's set and the three objectives identical to the oracle, on
+    random instances (unit to heavy chunks, so both DP kernels run) and on the
+    tiny and RAG workloads at full size."""
+    rng = np.random.default_rng(900)
+    cases = [wl.random_small(rng, int(rng.integers(1, 150)), int(rng.integers(1, 9)), 0,
+                             k_max=50, w_max=int(rng.choice([1, 2, 4, 6])), demand_max=40) for _ in range(12)]
+    cases += [wl.make(0), wl.make(1)]
+    for inst in cases:
+        with pp.Instance.from_workload(inst) as ppi:
+            gpl, gobj = pp.pp_safeguards(ppi)
+        opl, oobj = oracle_lib.safeguards(oracle_lib.Problem.from_instance(inst))
+        np.testing.assert_array_equal(gpl, opl)
+        np.testing.assert_array_equal(gobj, oobj)
+
+
+def test_plan_with_and_without_safeguards(pp, oracle_lib):
+    """A safeguard that beats every start is returned as candidate S + c, the
+    same as the oracle; without safeguards both return the best start; the
+    source-dependent objective has none (pp_safeguards refuses it)."""
+    rng = np.random.default_rng(901)
+    won = 0
+    for trial in range(16):
+        W = int(rng.integers(2, 6))
+        inst = wl.random_small(rng, int(rng.integers(2, 80)), W, 0, k_max=12, w_max=2, demand_max=30)
+        prob = oracle_lib.Problem.from_instance(inst)
+        S = int(rng.integers(1, 3))
+        with pp.Instance.from_workload(inst) as ppi:
+            g = pp.pp_plan_run(ppi, S, None, 1)
+            g0 = pp.pp_plan_run(ppi, S, None, 1, safeguards=False)
+        _compare_plans(g, oracle_lib.plan(prob, S, 1))
+        _compare_plans(g0, oracle_lib.plan(prob, S, 1, safeguards=False))
+        won += g.best_start >= S
+    assert won >= 1                       # the candidate path S + c is exercised
+    src = wl.random_small(rng, 30, 3, 1)
+    with pp.Instance.from_workload(src) as ppi:
+        with pytest.raises(pp.PPError):
+            pp.pp_safeguards(ppi)
+        assert pp.pp_plan_run(ppi, 2, None, 1).safeguard_objective == ()
 
 
 @pytest.mark.parametrize("mode", [0, 1])
