@@ -62,6 +62,7 @@ def _load():
             "or_default_orders": (ctypes.c_int, [P, i32, P]),
             "or_plan": (i32, [P, i32, P, i32, i32, P, P, P, P, P, P, ctypes.c_int, P]),
             "or_safeguards": (ctypes.c_int, [P, P, P]),
+            "or_replan": (ctypes.c_int, [P, P, i32, P, i32, i64, i64, i32, ctypes.c_int, P, P]),
             "or_worker_update": (i64, [P, i32, P, P, P]),
         }
         for name, (res, args) in sig.items():
@@ -226,6 +227,36 @@ def plan(prob: Problem, S: int, R: int, orders=None, threads: int | None = None,
     used = bool(safeguards) and prob.mode == 0
     return PlanResult(pl[:, :prob.n].copy(), int(obj.value), int(best), per, sw, acc, int(cells.value),
                       sg if used else None)
+
+
+@dataclass
+class ReplanResult:
+    placement: np.ndarray      # [W][n] uint8, the adopted target
+    incumbent_objective: int
+    new_objective: int
+    materialization_cost: int
+    break_even_requests: int   # -1 without a gain
+    adopted: bool
+
+
+def replan(prob: Problem, incumbent, S: int, R: int, epoch_requests: int, horizon_requests: int,
+           orders=None, threads: int | None = None, safeguards: bool = True) -> ReplanResult:
+    """Epoch update with the amortisation rule (Section IV-D, RQ5)."""
+    if threads is None:
+        threads = min(S, os.cpu_count() or 1)
+    inc = _c(incumbent, np.uint8)
+    assert inc.shape == (prob.W, prob.n)
+    pl = np.zeros((prob.W, max(prob.n, 1)), np.uint8)
+    out = np.zeros(5, np.int64)
+    op = None
+    if orders is not None:
+        orders = _c(orders, np.int32)
+        op = _ptr(orders)
+    r = _load().or_replan(prob.ref, _ptr(inc), int(S), op, int(R), int(epoch_requests), int(horizon_requests),
+                          int(threads), int(bool(safeguards)), _ptr(pl), _ptr(out))
+    if r != 0:
+        raise ValueError("parent array is not a forest")
+    return ReplanResult(pl[:, :prob.n].copy(), int(out[0]), int(out[1]), int(out[2]), int(out[3]), bool(out[4]))
 
 
 def worker_update(prob: Problem, h: int, placement):

@@ -33,6 +33,8 @@
  *                      Independent, Popularity, LocalDedup (Sections IV-C, V-A)
  *   or_plan            Algorithm 1 procedure PrefixPlace (greedy, refinement,
  *                      starts, and the safeguard candidates when asked for)
+ *   or_replan          epoch update with the amortisation rule (Section IV-D,
+ *                      RQ5 of Section V)
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -563,6 +565,59 @@ int32_t or_plan(const or_inst *I, int32_t S, const int32_t *orders, int32_t R, i
     if (cells_out) *cells_out = cells;
     free(th); free(st); free(T); free(order); free(next); free(ord);
     return best;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Epoch update (Section IV-D; the amortisation rule and break-even         */
+/* requests of RQ5, Section V).  Under the refreshed instance I (new demand) */
+/* the planner evaluates the incumbent T_old and a reoptimised target T_new  */
+/* (or_plan with S starts and R sweeps).  Making T_new resident costs, for   */
+/* every chunk b that worker m holds in T_new but not in T_old, what the     */
+/* materialisation rule of Section III-A charges requester m for b under    */
+/* the incumbent: the cheaper of recomputing and fetching from a worker that */
+/* holds b in T_old, or recomputing when none does.  G is a saving per epoch */
+/* of epoch_requests requests, so T_new is adopted iff                        */
+/*   (G(T_new) - G(T_old)) * horizon_requests > cost * epoch_requests,        */
+/* and break-even requests = ceil(cost * epoch_requests / (G_new - G_old))    */
+/* (-1 without a gain).  out5 = {G_old, G_new, cost, break_even, adopted};   */
+/* placement [W][n] out = the adopted target.  Returns 0, or -1 on an        */
+/* invalid tree.                                                              */
+/* ------------------------------------------------------------------------ */
+int or_replan(const or_inst *I, const uint8_t *incumbent, int32_t S, const int32_t *orders, int32_t R,
+              int64_t epoch_requests, int64_t horizon_requests, int32_t n_threads, int safeguards,
+              uint8_t *placement, int64_t *out5)
+{
+    int32_t n = I->n, W = I->W;
+    uint8_t *T = malloc((size_t)W * n + 1);
+    int64_t g_new = 0;
+    if (or_plan(I, S, orders, R, n_threads, T, &g_new, NULL, NULL, NULL, NULL, safeguards, NULL) < 0) {
+        free(T);
+        return -1;
+    }
+    int64_t g_old = or_objective(I, incumbent);
+    int64_t cost = 0;
+    for (int32_t m = 0; m < W; ++m)
+        for (int32_t b = 0; b < n; ++b) {
+            if (!HOLDS(T, I, m, b) || HOLDS(incumbent, I, m, b)) continue;
+            int64_t c = WCOST(I, m, b);                 /* recompute */
+            for (int32_t h = 0; h < W; ++h) {
+                if (h == m || !HOLDS(incumbent, I, h, b)) continue;
+                int64_t f = I->mode == 0 ? FREQ(I, m, b) : FPAIR(I, h, m, b);
+                c = imin64(c, f);                       /* fetch from an incumbent holder */
+            }
+            cost += c;
+        }
+    int64_t gain = g_new - g_old;
+    int64_t be = -1;
+    if (gain > 0) {
+        __int128 num = (__int128)cost * epoch_requests;
+        be = (int64_t)((num + gain - 1) / gain);
+    }
+    int adopt = gain > 0 && (__int128)gain * horizon_requests > (__int128)cost * epoch_requests;
+    memcpy(placement, adopt ? T : incumbent, (size_t)W * n);
+    out5[0] = g_old; out5[1] = g_new; out5[2] = cost; out5[3] = be; out5[4] = adopt;
+    free(T);
+    return 0;
 }
 
 /* One step of Algorithm 1 for a single worker, exposed so that one update of */

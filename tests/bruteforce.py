@@ -136,3 +136,24 @@ def best_set_by(parent, weight, k, value):
     order = preorder_positions(parent)
     cand = [s for s, v in zip(sets, vals) if v == best]
     return min(cand, key=lambda s: tuple(int(s[v]) for v in order)).astype(np.uint8)
+
+
+def materialisation_cost(inst, old, new) -> int:
+    """One-time cost of making `new` resident given `old`: for every chunk b a
+    worker m holds in `new` but not in `old`, requester m's Section III-A cost
+    of b under `old` (the cheaper of recomputing and fetching from an old
+    holder; recomputing when nobody holds it)."""
+    old = np.asarray(old, bool)
+    new = np.asarray(new, bool)
+    total = 0
+    for m in range(inst.W):
+        for b in range(inst.n):
+            if not new[m, b] or old[m, b]:
+                continue
+            w = int(inst.recompute[m, b])
+            holders = [h for h in range(inst.W) if old[h, b] and h != m]
+            if holders:
+                fetch = int(inst.transfer[m, b]) if inst.mode == 0 else min(int(inst.transfer[h, m, b]) for h in holders)
+                w = min(w, fetch)
+            total += w
+    return total

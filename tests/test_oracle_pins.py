@@ -402,6 +402,69 @@ def test_plan_never_worse_than_safeguards(oracle_lib):
         oracle_lib.safeguards(_prob(oracle_lib, src))
 
 
+# ------------------------------------------------------- epoch updates ---
+def _refreshed(rng, inst, kind):
+    """Demand after a shift: log-normal popularity noise, or a routing shift
+    that moves one worker's demand to another (cf. RQ5's transitions)."""
+    dem = inst.demand.copy()
+    if kind == 0:
+        dem = np.rint(dem * rng.lognormal(0.0, 1.0, dem.shape)).astype(np.int64)
+    else:
+        a, b = rng.choice(inst.W, 2, replace=False) if inst.W > 1 else (0, 0)
+        dem[[a, b]] = dem[[b, a]]
+    return wl.Instance(**{**inst.__dict__, "demand": dem})
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_replan_amortisation_rule(oracle_lib, mode):
+    """Section IV-D / RQ5: under refreshed demand the incumbent and the
+    reoptimised target are both evaluated; the one-time cost of the new chunks
+    is the Section III-A materialisation cost under the incumbent; the new
+    target is adopted iff gain * horizon > cost * epoch, and break-even
+    requests = ceil(cost * epoch / gain)."""
+    rng = np.random.default_rng(80 + mode)
+    seen = set()
+    for trial in range(24):
+        W = int(rng.integers(2, 5))
+        inst = wl.random_small(rng, int(rng.integers(3, 20)), W, mode, k_max=6, w_max=2, demand_max=40)
+        old = oracle_lib.plan(_prob(oracle_lib, inst), 2, 2, threads=1).placement
+        new_inst = _refreshed(rng, inst, trial % 2)
+        prob = _prob(oracle_lib, new_inst)
+        target = oracle_lib.plan(prob, 2, 2, threads=1).placement
+        epoch = 30000
+        r0 = oracle_lib.replan(prob, old, 2, 2, epoch, 1, threads=1)
+        assert r0.incumbent_objective == bf.materialisation_saving(new_inst, old)
+        assert r0.new_objective == bf.materialisation_saving(new_inst, target)
+        assert r0.materialization_cost == bf.materialisation_cost(new_inst, old, target)
+        gain, cost = r0.new_objective - r0.incumbent_objective, r0.materialization_cost
+        if gain <= 0:
+            assert r0.break_even_requests == -1 and not r0.adopted
+            np.testing.assert_array_equal(r0.placement, old)
+            seen.add("kept")
+            continue
+        be = r0.break_even_requests
+        assert be == -(-cost * epoch // gain)
+        for horizon in (max(be - 1, 0), be, be + 1, 10 * epoch):
+            r = oracle_lib.replan(prob, old, 2, 2, epoch, horizon, threads=1)
+            adopt = gain * horizon > cost * epoch
+            assert r.adopted == adopt
+            np.testing.assert_array_equal(r.placement, target if adopt else old)
+            seen.add(adopt)
+    assert {True, False} <= seen
+
+
+def test_replan_without_change_keeps_incumbent(oracle_lib):
+    """Unchanged demand and the same planner settings reproduce the incumbent:
+    no gain, no cost, nothing adopted."""
+    rng = np.random.default_rng(82)
+    inst = wl.random_small(rng, 40, 4, 0, k_max=10, w_max=2)
+    prob = _prob(oracle_lib, inst)
+    old = oracle_lib.plan(prob, 3, 3, threads=1).placement
+    r = oracle_lib.replan(prob, old, 3, 3, 30000, 10 ** 9, threads=1)
+    assert r.incumbent_objective == r.new_objective and r.materialization_cost == 0
+    assert not r.adopted and r.break_even_requests == -1
+
+
 def test_refinement_accepts_only_strict_improvements(oracle_lib):
     """Section IV-C: only strictly improving replacements are accepted, so a
     greedy result that is already coordinate-wise optimal ends after exactly
