@@ -360,6 +360,36 @@ pp_status pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *
  */
 pp_status pp_safeguards(pp_instance *inst, uint8_t *placement, int64_t *objective, void *stream);
 
+/* Outputs of pp_replan. */
+typedef struct {
+    int64_t incumbent_objective;   /* G(T_old) under the instance's (refreshed) demand */
+    int64_t new_objective;         /* G(T_new) of the reoptimised target */
+    int64_t materialization_cost;  /* one-time cost of the chunks T_new adds, microseconds */
+    int64_t break_even_requests;   /* ceil(cost * epoch_requests / (G_new - G_old)); -1 without a gain */
+    int32_t adopted;               /* 1: T_new returned; 0: the incumbent kept */
+} pp_replan_result;
+
+/*
+ * pp_replan -- epoch update with the amortisation rule (Section IV-D; the
+ * break-even requests of RQ5).  `inst` holds the refreshed demand.  The
+ * incumbent is scored under it, a reoptimised target is planned exactly as
+ * pp_plan_run does (n_starts, orders, max_rounds, stats as there), and the
+ * target's one-time cost is, for every chunk a worker holds in the target but
+ * not in the incumbent, the cheaper of recomputing it and fetching it from a
+ * worker that holds it in the incumbent (recomputing when none does) -- the
+ * Section III-A materialisation rule applied to the incumbent.  G is a saving
+ * per epoch of `epoch_requests` requests, so the target is adopted iff
+ *   (G_new - G_old) * horizon_requests > cost * epoch_requests.
+ *   incumbent     host [W][n] by node id, nonzero = resident
+ *   placement     host [W][n] out: the target if adopted, else the incumbent
+ *   result        host out
+ * Synchronous.  Errors: PP_EINVAL (epoch_requests <= 0, horizon_requests < 0,
+ * null pointers, and those of pp_plan_run), PP_ENOMEM, PP_ECUDA, device status.
+ */
+pp_status pp_replan(pp_instance *inst, const uint8_t *incumbent, int32_t n_starts, const int32_t *orders,
+                    int32_t max_rounds, int64_t epoch_requests, int64_t horizon_requests,
+                    uint8_t *placement, pp_replan_result *result, pp_plan_stats *stats, void *stream);
+
 /* Thread-local description of the last failure in this thread ("" if none). */
 const char *pp_last_error(void);
 

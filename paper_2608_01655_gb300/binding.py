@@ -68,6 +68,7 @@ _SIGS = {
     "pp_default_orders": [_P, _i32, _P, _P],
     "pp_probe_read": [_P, ctypes.c_size_t, _i32, _P, _P],
     "pp_safeguards": [_P, _P, _P, _P],
+    "pp_replan": [_P, _P, _i32, _P, _i32, _i64, _i64, _P, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -310,3 +311,40 @@ def pp_safeguards(inst: Instance, stream=None):
     obj = np.zeros(3, np.int64)
     _check(_lib.pp_safeguards(inst.handle, _host(pl), _host(obj), _stream(stream)))
     return pl[:, :, :inst.n].copy(), obj
+
+
+class ReplanStruct(ctypes.Structure):
+    _fields_ = [("incumbent_objective", _i64), ("new_objective", _i64), ("materialization_cost", _i64),
+                ("break_even_requests", _i64), ("adopted", _i32)]
+
+
+@dataclass
+class ReplanResult:
+    placement: np.ndarray
+    incumbent_objective: int
+    new_objective: int
+    materialization_cost: int
+    break_even_requests: int
+    adopted: bool
+
+
+def pp_replan(inst: Instance, incumbent, n_starts: int, max_rounds: int, epoch_requests: int,
+              horizon_requests: int, orders=None, safeguards: bool = True, stream=None) -> ReplanResult:
+    """Epoch update with the amortisation rule; incumbent [W][n] uint8 (host)."""
+    inc = _np(incumbent, np.uint8)
+    if inc.shape != (inst.W, inst.n):
+        raise ValueError("incumbent must be [W][n]")
+    pl = np.zeros((inst.W, max(inst.n, 1)), np.uint8)
+    res = ReplanStruct()
+    st = PlanStats()
+    st.no_safeguards = int(not safeguards)
+    op = None
+    if orders is not None:
+        orders = _np(orders, np.int32)
+        if orders.shape != (int(n_starts), inst.W):
+            raise ValueError("orders must be [n_starts][W]")
+        op = _host(orders)
+    _check(_lib.pp_replan(inst.handle, _host(inc), int(n_starts), op, int(max_rounds), int(epoch_requests),
+                          int(horizon_requests), _host(pl), ctypes.byref(res), ctypes.byref(st), _stream(stream)))
+    return ReplanResult(pl[:, :inst.n].copy(), int(res.incumbent_objective), int(res.new_objective),
+                        int(res.materialization_cost), int(res.break_even_requests), bool(res.adopted))

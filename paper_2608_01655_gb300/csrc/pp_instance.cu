@@ -224,12 +224,15 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     cudaFree(inst->d_delta);
     cudaFree(inst->d_own);
     cudaFree(inst->d_pop);
+    cudaFree(inst->d_rec);
+    cudaFree(inst->d_tr);
     cudaFree(inst->d_g);
     cudaFree(inst->d_status);
     free_scratch(inst->stack);
     free_scratch(inst->plan);
     free_scratch(inst->plan_bits);
     free_scratch(inst->sg);
+    free_scratch(inst->rp);
     cudaSetDevice(cur);
     delete inst;
     return PP_OK;
@@ -315,10 +318,13 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     PP_CUDA(cudaMalloc(&inst->d_status, sizeof(int32_t)));
     PP_CUDA(cudaMemsetAsync(inst->d_status, 0, sizeof(int32_t), st));
 
-    int64_t *d_dem = nullptr, *d_rec = nullptr, *d_tr = nullptr;
+    // recompute and transfer costs stay resident (by node id) for the epoch
+    // update's materialisation cost; demand is needed only here
+    int64_t *d_dem = nullptr;
     if ((s = upload(&d_dem, demand, Wn, st))) return s;
-    if ((s = upload(&d_rec, recompute, Wn, st))) { cudaFree(d_dem); return s; }
-    if ((s = upload(&d_tr, transfer, tn, st))) { cudaFree(d_dem); cudaFree(d_rec); return s; }
+    if ((s = upload(&inst->d_rec, recompute, Wn, st))) { cudaFree(d_dem); return s; }
+    if ((s = upload(&inst->d_tr, transfer, tn, st))) { cudaFree(d_dem); return s; }
+    int64_t *const d_rec = inst->d_rec, *const d_tr = inst->d_tr;
     cudaError_t e = cudaSuccess;
     int blocks = (int)((n + 255) / 256);
     if (blocks > 4 * inst->sm_count) blocks = 4 * inst->sm_count;
@@ -341,8 +347,6 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     cudaFree(d_dem);
-    cudaFree(d_rec);
-    cudaFree(d_tr);
     if (e != cudaSuccess) return cuda_fail(e, "gain precompute");
     return PP_OK;
 }

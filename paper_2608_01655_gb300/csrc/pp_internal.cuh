@@ -131,12 +131,15 @@ struct pp_instance {
     int64_t *d_delta = nullptr;         // mode 0: [n]    Delta(b)     (Eq. 3)
     int64_t *d_own = nullptr;           // mode 0: [W][n] Lambda_m(b) [w_m(b) - f_m(b)]_+ (own first-copy gain)
     int64_t *d_pop = nullptr;           // mode 0: [W][n] Lambda_m(b)
+    int64_t *d_rec = nullptr;           // [W][n] w_m(b) by node id
+    int64_t *d_tr = nullptr;            // by node id: mode 0 [W][n] f_m(b), mode 1 [W][W][n] f_{m<-h}(b)
     int64_t *d_g = nullptr;             // mode 1: [W][W][n] Lambda_m(b) q_{m<-h}(b) at [h][m][i] (Eq. 5)
     int32_t *d_status = nullptr;        // device status word
     pp::Scratch stack;                  // skip-row stack spill of pp_tree_dp
     pp::Scratch plan;                   // pp_plan_run working set
     pp::Scratch plan_bits;              // pp_plan_run decision bits
     pp::Scratch sg;                     // safeguard candidates' working set
+    pp::Scratch rp;                     // epoch update working set
 };
 
 namespace pp {
@@ -193,6 +196,9 @@ pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, con
 // holder masks [3][n] in preorder (device, in inst->sg, valid until the next
 // call) and their objectives (host [3]).  Adds its kernel launches and DP
 // cells to the counters.
+pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t R, uint8_t *placement,
+                    int64_t *objective, pp_plan_stats *stats, cudaStream_t st, bool orders_only = false);
+
 pp_status safeguards_impl(pp_instance *inst, cudaStream_t st, const uint32_t **masks, int64_t *obj,
                           int *launches, int64_t *cells, int *dp_launches);
 

@@ -80,9 +80,9 @@ static pp_status plan_buffers(pp_instance *inst, int B, PlanBuffers *pb)
     return PP_OK;
 }
 
-static pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t R,
-                           uint8_t *placement, int64_t *objective, pp_plan_stats *stats,
-                           cudaStream_t st, bool orders_only = false)
+pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t R,
+                    uint8_t *placement, int64_t *objective, pp_plan_stats *stats,
+                    cudaStream_t st, bool orders_only)
 {
     const int32_t n = inst->n, W = inst->W;
     int launches = 0;

@@ -223,6 +223,46 @@ def test_plan_parity_workloads(pp, oracle_lib, cfg):
     assert g.dp_cells == o.cells
 
 
+def _shifted(rng, inst, kind):
+    dem = inst.demand.copy()
+    if kind == 0:
+        dem = np.rint(dem * rng.lognormal(0.0, 1.0, dem.shape)).astype(np.int64)
+    else:
+        a, b = rng.choice(inst.W, 2, replace=False)
+        dem[[a, b]] = dem[[b, a]]
+    return wl.Instance(**{**inst.__dict__, "demand": dem})
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_replan_matches_oracle(pp, oracle_lib, mode):
+    """Epoch update (Section IV-D, RQ5): incumbent and new objectives,
+    materialisation cost, break-even requests, the adoption decision and the
+    returned placement identical to the oracle, for several horizons."""
+    rng = np.random.default_rng(950 + mode)
+    cases = [wl.random_small(rng, int(rng.integers(2, 120)), int(rng.integers(2, 7)), mode, k_max=30,
+                             w_max=2, demand_max=40) for _ in range(6)]
+    if mode == 0:
+        cases.append(wl.make(1))
+    for t, inst in enumerate(cases):
+        S, R = min(inst.starts, 4) if inst.starts > 1 else 2, 2
+        old = oracle_lib.plan(oracle_lib.Problem.from_instance(inst), S, R).placement
+        new = _shifted(rng, inst, t % 2)
+        prob = oracle_lib.Problem.from_instance(new)
+        o = oracle_lib.replan(prob, old, S, R, 30000, 1)
+        horizons = [1, 10 ** 9] + ([o.break_even_requests, o.break_even_requests + 1]
+                                   if o.break_even_requests > 0 else [])
+        with pp.Instance.from_workload(new) as ppi:
+            for h in horizons:
+                g = pp.pp_replan(ppi, old, S, R, 30000, h)
+                o = oracle_lib.replan(prob, old, S, R, 30000, h)
+                assert (g.incumbent_objective, g.new_objective, g.materialization_cost, g.break_even_requests,
+                        g.adopted) == (o.incumbent_objective, o.new_objective, o.materialization_cost,
+                                       o.break_even_requests, o.adopted)
+                np.testing.assert_array_equal(g.placement, o.placement)
+            with pytest.raises(pp.PPError):
+                pp.pp_replan(ppi, old, S, R, 0, 1)
+
+
 def _random_feasible_placement(rng, inst, frac):
     """Parent-closed, within-budget placement grown top-down (a plausible
     mid-refinement state to sample one update from)."""
