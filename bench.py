@@ -268,6 +268,41 @@ def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, s
     }
 
 
+def _extras(pp, torch, wl, inst, res):
+    """Timings of the steps next to the plan (outside the timed region):
+    the requester-side safeguard candidates on the RAG workload, and one epoch
+    update of the paper-scale plan after a popularity shift (log-normal
+    sigma = 0.5 on every demand entry, as in RQ5)."""
+    out = {}
+    rag = wl.make(1)
+    with pp.Instance.from_workload(rag) as ppr:
+        pp.pp_safeguards(ppr)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        _, sg_obj = pp.pp_safeguards(ppr)
+        t_sg = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        r1 = pp.pp_plan_run(ppr, rag.starts, None, rag.rounds)
+        t_plan = time.perf_counter() - t0
+    out["safeguards"] = {"workload": rag.name, "ms": 1000 * t_sg, "objectives": [int(x) for x in sg_obj],
+                         "plan_ms_with_safeguards": 1000 * t_plan, "plan_objective": r1.objective,
+                         "plan_best_candidate": r1.best_start}
+    rng = np.random.default_rng(2026)
+    dem = np.rint(inst.demand * rng.lognormal(0.0, 0.5, inst.demand.shape)).astype(np.int64)
+    shifted = wl.Instance(**{**inst.__dict__, "demand": dem})
+    with pp.Instance.from_workload(shifted) as pps:
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        rr = pp.pp_replan(pps, res.placement, inst.starts, inst.rounds, wl.REQUESTS_PER_EPOCH,
+                          wl.REQUESTS_PER_EPOCH)
+        t_rp = time.perf_counter() - t0
+    out["epoch_update"] = {"workload": inst.name, "shift": "popularity, log-normal sigma 0.5", "ms": 1000 * t_rp,
+                           "incumbent_objective": rr.incumbent_objective, "new_objective": rr.new_objective,
+                           "materialization_cost_us": rr.materialization_cost,
+                           "break_even_requests": rr.break_even_requests, "adopted_at_one_epoch": rr.adopted}
+    return out
+
+
 def run_native(args):
     import torch
     world, rank, local = _dist()
@@ -393,6 +428,8 @@ def run_native(args):
         e2e_total = float(t.item())
     e2e_value = world * cells_per_plan * args.steps / e2e_total
 
+    extras = _extras(pp, torch, wl, inst, res) if rank == 0 else None
+
     # ---- candidates of all ranks compared once (outside the timed region) ---
     best_obj, best_start = res.objective, res.best_start
     if world > 1:
@@ -433,6 +470,7 @@ def run_native(args):
             "update_ms": sum(phase_sum) / (nl * args.steps),
             "update_note": "one batched worker update (marginals + tree DP + traceback/accept) of all starts",
             "probes": probes,
+            "next_steps": extras,
             "dp_geometry": pp.pp_dp_geometry(ppi, S, k),
         }
         print(json.dumps(line), flush=True)

@@ -76,6 +76,10 @@ typedef struct {
     int32_t no_safeguards;         /* in: nonzero = leave out the safeguard candidates */
     int64_t safeguard_objective[3];/* out: Independent, Popularity, LocalDedup objectives
                                       (requester-side only; else 0) */
+    int32_t marginals;             /* in, source-dependent only: 0 automatic, 1 scan each
+                                      chunk's holders, 2 keep top-2 holder tables per start
+                                      (Section IV-C); results are identical */
+    int32_t used_top2;             /* out: 1 if the top-2 tables were used */
 } pp_plan_stats;
 
 /*

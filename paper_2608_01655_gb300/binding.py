@@ -45,7 +45,7 @@ class PlanStats(ctypes.Structure):
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
                 ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
                 ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32), ("no_safeguards", _i32),
-                ("safeguard_objective", ctypes.c_int64 * 3)]
+                ("safeguard_objective", ctypes.c_int64 * 3), ("marginals", _i32), ("used_top2", _i32)]
 
 
 _SIGS = {
@@ -243,10 +243,12 @@ class PlanResult:
     dp_rows_swept: int = 0
     dp_launches: int = 0
     safeguard_objective: tuple = ()     # Independent, Popularity, LocalDedup (requester-side)
+    used_top2: bool = False             # source-dependent marginals from top-2 holder tables
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
-                time_phases: bool = False, safeguards: bool = True) -> PlanResult:
+                time_phases: bool = False, safeguards: bool = True, marginals: int = 0) -> PlanResult:
+    """marginals (source-dependent): 0 automatic, 1 holder scan, 2 top-2 tables."""
     S, W, n = int(n_starts), inst.W, inst.n
     placement = np.zeros((W, max(n, 1)), np.uint8)
     obj = _i64(0)
@@ -257,6 +259,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
     st = PlanStats(per.ctypes.data, sw.ctypes.data, acc.ctypes.data, used.ctypes.data, 0, 0, 0, 0, 0,
                    int(bool(time_phases)))
     st.no_safeguards = int(not safeguards)
+    st.marginals = int(marginals)
     op = None
     if orders is not None:
         orders = _np(orders, np.int32)
@@ -269,7 +272,8 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                       int(st.dp_count), int(st.dp_cells), int(st.kernel_launches),
                       tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept),
                       int(st.dp_launches),
-                      tuple(int(x) for x in st.safeguard_objective) if safeguards and inst.mode == 0 else ())
+                      tuple(int(x) for x in st.safeguard_objective) if safeguards and inst.mode == 0 else (),
+                      bool(st.used_top2))
 
 
 def pp_test_inject(kind: int, value: int):

@@ -233,6 +233,7 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     free_scratch(inst->plan_bits);
     free_scratch(inst->sg);
     free_scratch(inst->rp);
+    free_scratch(inst->top2);
     cudaSetDevice(cur);
     delete inst;
     return PP_OK;

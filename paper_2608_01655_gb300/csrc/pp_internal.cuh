@@ -140,6 +140,7 @@ struct pp_instance {
     pp::Scratch plan_bits;              // pp_plan_run decision bits
     pp::Scratch sg;                     // safeguard candidates' working set
     pp::Scratch rp;                     // epoch update working set
+    pp::Scratch top2;                   // top-2 holder tables of the planner
 };
 
 namespace pp {
@@ -174,6 +175,19 @@ pp_status launch_marginals(pp_instance *inst, int batch, const int32_t *worker,
 
 pp_status launch_objective(pp_instance *inst, int batch, const uint32_t *mask,
                            const uint8_t *chosen, int64_t *obj, cudaStream_t st);
+
+// Top-2 holder tables of the source-dependent marginals, per start (batch item):
+// v1, v2, l1 [batch][W][n] and the pre-update bit of the current worker [batch][n].
+struct Top2 {
+    int64_t *v1 = nullptr;
+    int64_t *v2 = nullptr;
+    int8_t *l1 = nullptr;
+    uint8_t *oldbit = nullptr;
+};
+pp_status launch_marginals_top2(pp_instance *inst, int batch, const int32_t *prev_worker, const int32_t *worker,
+                                const uint32_t *mask, const int32_t *item_active, const Top2 &t2,
+                                int64_t *profit, int64_t *oldsum, cudaStream_t st);
+
 
 // Traceback of pp_tree_dp's bits.  With mask == nullptr it writes chosen[]
 // bytes by node id (ABI); otherwise it is the planner's accept-and-update

@@ -14,6 +14,10 @@
 
 namespace pp {
 
+// automatic choice of the top-2 marginals: whenever the tables (17 bytes per
+// start, requester and chunk) fit in this much device memory
+constexpr size_t kTop2MaxBytes = (size_t)16 << 30;
+
 // per-sweep bookkeeping: a start that accepted nothing is done
 __global__ void k_sweep_end(int S, int32_t *active, const int32_t *improved, int32_t *sweeps)
 {
@@ -197,12 +201,39 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
 
     int dp_count = standalone_cells ? W : 0;
     int64_t cells = standalone_cells;
+    // source-dependent marginals: scan each chunk's holders, or keep top-2
+    // holder tables (Section IV-C); automatic = top-2 when the tables fit
+    const int mreq = stats ? stats->marginals : 0;
+    if (mreq < 0 || mreq > 2) return fail(PP_EINVAL, "stats->marginals must be 0, 1 or 2");
+    const bool use_top2 = inst->mode == PP_TRANSFER_SOURCE && n > 0 &&
+                          (mreq == 2 || (mreq == 0 && (size_t)S * W * n * 17 <= kTop2MaxBytes));
+    Top2 t2;
+    if (use_top2) {
+        const size_t tw = (size_t)S * W * n, a = 255;
+        const size_t b1 = (8 * tw + a) & ~a, b2 = b1 + ((8 * tw + a) & ~a), b3 = b2 + ((tw + a) & ~a);
+        if ((s = ensure_scratch(inst->top2, b3 + (size_t)S * n))) return s;
+        char *base = reinterpret_cast<char *>(inst->top2.ptr);
+        t2.v1 = reinterpret_cast<int64_t *>(base);
+        t2.v2 = reinterpret_cast<int64_t *>(base + b1);
+        t2.l1 = reinterpret_cast<int8_t *>(base + b2);
+        t2.oldbit = reinterpret_cast<uint8_t *>(base + b3);
+        PP_CUDA(cudaMemsetAsync(base, 0, b2, st));                 // v1 = v2 = 0: no holders yet
+        PP_CUDA(cudaMemsetAsync(t2.l1, 0xFF, tw, st));             // l1 = -1
+    }
+    const int32_t *prev_wk = nullptr;     // top-2: worker of the previous step, per start
     auto step = [&](int t, int greedy) -> pp_status {
         const int32_t *wk = pb.work + (size_t)t * B;
         const int32_t *kb = pb.kbud + (size_t)t * B;
         pp_status r;
         if ((r = mark())) return r;
-        if ((r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st))) return r;
+        if (use_top2) {
+            // the previous step's change is folded into this step's marginal pass
+            r = launch_marginals_top2(inst, S, prev_wk, wk, pb.mask, pb.active, t2, pb.profit, pb.oldsum, st);
+            prev_wk = wk;
+        } else {
+            r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st);
+        }
+        if (r) return r;
         if ((r = mark())) return r;
         if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, work, st, maxk, rows_kept)))
             return r;
@@ -303,6 +334,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         stats->dp_rows_swept = (int64_t)rows_swept;
         stats->dp_launches = dp_launches;
         for (int c = 0; c < 3; ++c) stats->safeguard_objective[c] = so[c];
+        stats->used_top2 = use_top2;
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
         for (size_t x = 0; x + 3 < ev.v.size(); x += 4) {
             float a = 0.f, b = 0.f, c = 0.f;

@@ -223,6 +223,32 @@ def test_plan_parity_workloads(pp, oracle_lib, cfg):
     assert g.dp_cells == o.cells
 
 
+def test_plan_top2_marginals(pp, oracle_lib):
+    """Source-dependent plans with the marginals taken from top-2 holder tables
+    (Section IV-C) and from scanning the holders: both identical to the oracle,
+    including dense holder sets (budgets close to n) and ties in g."""
+    rng = np.random.default_rng(960)
+    cases = []
+    for t in range(8):
+        n = int(rng.integers(2, 150))
+        W = int(rng.integers(2, 9))
+        inst = wl.random_small(rng, n, W, 1, k_max=max(2, n), w_max=2, demand_max=20)
+        if t % 3 == 0:                                    # many equal gains: ties in the tables
+            inst = wl.Instance(**{**inst.__dict__, "transfer": np.minimum(inst.transfer, 3),
+                                  "recompute": np.minimum(inst.recompute, 5)})
+        cases.append(inst)
+    cases.append(wl.make(2))
+    for inst in cases:
+        prob = oracle_lib.Problem.from_instance(inst)
+        S = min(inst.starts, 3) if inst.starts > 1 else 2
+        o = oracle_lib.plan(prob, S, 3)
+        with pp.Instance.from_workload(inst) as ppi:
+            for mode in (1, 2):
+                g = pp.pp_plan_run(ppi, S, None, 3, marginals=mode)
+                assert g.used_top2 == (mode == 2)
+                _compare_plans(g, o)
+
+
 def _shifted(rng, inst, kind):
     dem = inst.demand.copy()
     if kind == 0:
