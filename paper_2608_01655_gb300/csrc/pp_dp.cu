@@ -389,9 +389,14 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             uint32_t wb8[C];
 #pragma unroll
             for (int c = 0; c < C; ++c) wb8[c] = 0;
+            // the sub-block's profits, read before any skip-row stack store
+            // (which the compiler cannot move a later shared load above)
+            int64_t pv[kSub];
+#pragma unroll
+            for (int u = 0; u < kSub; ++u) pv[u] = my_p[s8 + u];
             // one row of Eq. 9 for this warp's columns; STACK: the row may push or pop
             auto row = [&](const int u, const bool STACK) {
-                const int64_t p = my_p[s8 + u];
+                const int64_t p = pv[u];
                 // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
                 // (the first warp's sv is all zero: column 0 of every row is 0)
                 int64_t bnd[WMAX];
