@@ -659,12 +659,14 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 // mark b_i, j -= w_i and go to the next kept row; skip -> go to next(i); stop
 // at i = n or j = 0.  In kept-row order a take always moves from kept index t
 // to t - 1 (the next kept row in preorder, since a pruned interior is all
-// "skip"), and a skip moves to skip[t].  One warp walks and speculates each
-// round on two take-runs: lanes 0-15 on the run that starts at t, lanes 16-31
-// on the run that starts at u = skip[t] (used when row t itself is skipped);
-// with skip and skip2 tables every address of the round is known up front
-// (after the suffix weights for weighted trees).  A round resolves an optional
-// skip of t, one take-run and the skip that ends it.
+// "skip"), and a skip moves to skip[t].  The walk is monotone in t and j, so
+// one warp reads it tile by tile: a tile is 64 kept rows x 32 columns, whose
+// decision bits are 64 words (one word holds 32 rows of one column), loaded
+// together with the tile's skip targets, positions and suffix weights in one
+// round of independent loads.  Inside the tile every step is register work:
+// lane l tests row t - l at the column reached after taking rows t..t-l+1, a
+// ballot gives the take-run, and the row that ends it is the skip.  A step
+// that leaves the tile (rows below it, or columns left of it) loads the next.
 // Planner mode (acc.mask != nullptr): the update is accepted in the greedy
 // pass, or in refinement iff D[0][k] > sum of p_h over the current T_h
 // (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
@@ -705,65 +707,85 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     const int nblk = (n + 31) / 32;
     const uint32_t *Bi = w.bits + (size_t)item * P * (size_t)nblk * C * 32;
     const int32_t *rl = w.rowlist + (size_t)item * n;
-    const int32_t *sk = w.skip + (size_t)item * n, *sk2 = w.skip2 + (size_t)item * n;
+    const int32_t *sk = w.skip + (size_t)item * n;
     const int32_t *ws = w.wsuf + (size_t)item * (n + 1);
     const int nk = w.nkept[item];
-    auto bit = [&](int row, int col) -> uint32_t {           // decision of kept row `row`, column col >= 1
+    auto word_at = [&](int blk, int col) -> uint32_t {       // bits of rows blk*32.. at column col >= 1
         const int q = col - 1;
         const int tt = q / C, c = q - tt * C;
-        const uint32_t word = Bi[(((size_t)(tt >> 5) * nblk + (row >> 5)) * C + c) * 32 + (tt & 31)];
-        return (word >> (row & 31)) & 1u;
+        return Bi[(((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31)];
     };
     int t = nk - 1;                 // row of position 0 (the first root): swept last
-    int u = nk > 0 ? sk[t] : -1;
-    const int half = lane >> 4, l = lane & 15;
-    for (int guard = 0; guard <= n && t >= 0 && j > 0; ++guard) {
-        // lane (half, l): row `l` steps into the take-run from t (half 0) or u (half 1)
-        const int base = half ? u : t;
-        const int row = base - l;
-        const bool live = base >= 0 && row >= 0;
-        int col = j;
-        if (live && l > 0) col = unit_weights ? j - l : j - (ws[row + 1] - ws[base + 1]);
-        const bool take = live && col > 0 && bit(row, col);
-        const int pos = live ? rl[row] : -1;
-        const int s1 = live ? sk[row] : -1, s2 = live ? sk2[row] : -1;
-        const int wrow = live ? (unit_weights ? 1 : ws[row] - ws[row + 1]) : 0;   // w of kept row `row`
-        const uint32_t tm = __ballot_sync(kFull, take);
-        int h0;                                           // the half that continues the walk
-        if (tm & 1u) {
-            h0 = 0;
-        } else {
-            if (u < 0) break;                             // t skipped and next(t) = n: done
-            if (!(tm & 0x10000u)) {                       // u skipped too
-                const int nt = __shfl_sync(kFull, s1, 16), nu = __shfl_sync(kFull, s2, 16);
-                t = nt;
-                u = nu;
+    for (int guard = 0; guard <= 2 * n + 2 && t >= 0 && j > 0; ++guard) {
+        // ---- load the tile holding (t, j): rows r0..r0+63, columns j0-31..j0
+        const int r0 = t & ~63, j0 = j;
+        const int colx = j0 - lane;
+        uint32_t wlo = 0, whi = 0;
+        if (colx >= 1) {
+            wlo = word_at(r0 >> 5, colx);
+            if (r0 + 32 < nk) whi = word_at((r0 >> 5) + 1, colx);
+        }
+        int sklo = -1, skhi = -1, rllo = 0, rlhi = 0, wslo = 0, wshi = 0;
+        if (r0 + lane < nk) {
+            sklo = sk[r0 + lane];
+            rllo = rl[r0 + lane];
+            if (!unit_weights) wslo = ws[r0 + lane];
+        }
+        if (r0 + 32 + lane < nk) {
+            skhi = sk[r0 + 32 + lane];
+            rlhi = rl[r0 + 32 + lane];
+            if (!unit_weights) wshi = ws[r0 + 32 + lane];
+        }
+        const int wstop = unit_weights ? 0 : ws[min(r0 + 64, nk)];
+        // suffix weight of kept row r in r0..r0+64 (register shuffles; every lane calls it)
+        auto wsat = [&](int r) -> int {
+            const int lr = r - r0;
+            const int a = __shfl_sync(kFull, wslo, lr & 31), b = __shfl_sync(kFull, wshi, lr & 31);
+            return lr >= 64 ? wstop : (lr < 32 ? a : b);
+        };
+        // ---- walk inside the tile
+        while (t >= r0 && j > 0 && j > j0 - 32) {
+            const int row = t - lane;
+            const int lr = (row - r0) & 63;
+            int col, coln;
+            if (unit_weights) {
+                col = j - lane;
+                coln = col - 1;
+            } else {
+                const int wt = wsat(t + 1), wr = wsat(row + 1), wr0 = wsat(row);
+                col = j - (wr - wt);
+                coln = j - (wr0 - wt);
+            }
+            const bool valid = row >= r0 && col >= 1 && col > j0 - 32;
+            const int src = (j0 - col) & 31;
+            const uint32_t wa = __shfl_sync(kFull, wlo, src), wb = __shfl_sync(kFull, whi, src);
+            const uint32_t word = lr < 32 ? wa : wb;
+            const bool take = valid && ((word >> (lr & 31)) & 1u);
+            const uint32_t tm = __ballot_sync(kFull, take);
+            const int L = tm == kFull ? 32 : __ffs(~tm) - 1;    // rows t..t-L+1 are taken
+            const int pa = __shfl_sync(kFull, rllo, lr & 31), pb = __shfl_sync(kFull, rlhi, lr & 31);
+            const int sa = __shfl_sync(kFull, sklo, lr & 31), sb = __shfl_sync(kFull, skhi, lr & 31);
+            if (lane < L) {
+                const int pos = lr < 32 ? pa : pb;
+                if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
+                else chosen[(size_t)item * n + order[pos]] = 1;
+            }
+            if (L == 32) {                                    // 32 takes: continue after the last
+                j = __shfl_sync(kFull, coln, 31);
+                t -= 32;
                 continue;
             }
-            h0 = 1;
+            const int vL = __shfl_sync(kFull, (int)valid, L);
+            const int colL = __shfl_sync(kFull, col, L);
+            const int skL = __shfl_sync(kFull, lr < 32 ? sa : sb, L);
+            j = colL;
+            if (vL) {
+                t = skL;                                      // row t-L is skipped: next(i), -1 = past n
+            } else {
+                t -= L;                                       // (t-L, colL) lies outside the tile
+                break;
+            }
         }
-        const uint32_t run = (tm >> (16 * h0)) & 0xFFFFu;
-        const int l0 = __ffs(~run) - 1 < 16 ? __ffs(~run) - 1 : 16;   // first lane of the half not taken
-        if (half == h0 && l < l0) {
-            if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
-            else chosen[(size_t)item * n + order[pos]] = 1;
-        }
-        const int src = 16 * h0 + (l0 < 16 ? l0 : 15);
-        const int ecol = __shfl_sync(kFull, col, src);
-        const int erow = __shfl_sync(kFull, row, src);
-        const int es1 = __shfl_sync(kFull, s1, src), es2 = __shfl_sync(kFull, s2, src);
-        const int ew = __shfl_sync(kFull, wrow, src);
-        const int ebase = h0 ? u : t;
-        if (l0 == 16) {                                   // 16 takes: continue after the last
-            t = ebase - 16;
-            j = ecol - ew;
-            u = t >= 0 ? sk[t] : -1;
-            continue;
-        }
-        if (erow < 0 || ecol <= 0) break;                 // ran past position n-1 or out of slots
-        t = es1;                                          // row erow is skipped
-        u = es2;
-        j = ecol;
     }
 }
 
