@@ -672,6 +672,8 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 // (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
 // replaces bit h of the holder masks by the traced set.
 // ===========================================================================
+constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (a multiple of 32)
+
 __global__ void __launch_bounds__(256)
 k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
@@ -716,37 +718,42 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
         return Bi[(((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31)];
     };
     int t = nk - 1;                 // row of position 0 (the first root): swept last
+    constexpr int TB = kTraceTileRows / 32;                   // 32-row blocks per tile
     for (int guard = 0; guard <= 2 * n + 2 && t >= 0 && j > 0; ++guard) {
-        // ---- load the tile holding (t, j): rows r0..r0+63, columns j0-31..j0
-        const int r0 = t & ~63, j0 = j;
+        // ---- load the tile holding (t, j): rows r0..r0+TB*32-1, columns j0-31..j0
+        const int r0 = t & ~(kTraceTileRows - 1), j0 = j;
         const int colx = j0 - lane;
-        uint32_t wlo = 0, whi = 0;
-        if (colx >= 1) {
-            wlo = word_at(r0 >> 5, colx);
-            if (r0 + 32 < nk) whi = word_at((r0 >> 5) + 1, colx);
+        uint32_t wv[TB];
+        int skv[TB], rlv[TB], wsv[TB];
+#pragma unroll
+        for (int x = 0; x < TB; ++x) {
+            const int r = r0 + 32 * x + lane;
+            wv[x] = (colx >= 1 && r0 + 32 * x < nk) ? word_at((r0 >> 5) + x, colx) : 0u;
+            skv[x] = r < nk ? sk[r] : -1;
+            rlv[x] = r < nk ? rl[r] : 0;
+            wsv[x] = (!unit_weights && r < nk) ? ws[r] : 0;
         }
-        int sklo = -1, skhi = -1, rllo = 0, rlhi = 0, wslo = 0, wshi = 0;
-        if (r0 + lane < nk) {
-            sklo = sk[r0 + lane];
-            rllo = rl[r0 + lane];
-            if (!unit_weights) wslo = ws[r0 + lane];
-        }
-        if (r0 + 32 + lane < nk) {
-            skhi = sk[r0 + 32 + lane];
-            rlhi = rl[r0 + 32 + lane];
-            if (!unit_weights) wshi = ws[r0 + 32 + lane];
-        }
-        const int wstop = unit_weights ? 0 : ws[min(r0 + 64, nk)];
-        // suffix weight of kept row r in r0..r0+64 (register shuffles; every lane calls it)
+        const int wstop = unit_weights ? 0 : ws[min(r0 + kTraceTileRows, nk)];
+        // a register of block lr / 32 of the lane lr % 32 (every lane calls it)
+        auto pick = [&](const auto &v, int lr, int from) {
+            int out = 0;
+#pragma unroll
+            for (int x = 0; x < TB; ++x) {
+                const int y = __shfl_sync(kFull, (int)v[x], from);
+                out = (lr >> 5) == x ? y : out;
+            }
+            return out;
+        };
+        // suffix weight of kept row r in r0..r0+TB*32
         auto wsat = [&](int r) -> int {
             const int lr = r - r0;
-            const int a = __shfl_sync(kFull, wslo, lr & 31), b = __shfl_sync(kFull, wshi, lr & 31);
-            return lr >= 64 ? wstop : (lr < 32 ? a : b);
+            const int y = pick(wsv, lr, lr & 31);
+            return lr >= kTraceTileRows ? wstop : y;
         };
         // ---- walk inside the tile
         while (t >= r0 && j > 0 && j > j0 - 32) {
             const int row = t - lane;
-            const int lr = (row - r0) & 63;
+            const int lr = (row - r0) & (kTraceTileRows - 1);
             int col, coln;
             if (unit_weights) {
                 col = j - lane;
@@ -757,16 +764,13 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
                 coln = j - (wr0 - wt);
             }
             const bool valid = row >= r0 && col >= 1 && col > j0 - 32;
-            const int src = (j0 - col) & 31;
-            const uint32_t wa = __shfl_sync(kFull, wlo, src), wb = __shfl_sync(kFull, whi, src);
-            const uint32_t word = lr < 32 ? wa : wb;
+            const uint32_t word = (uint32_t)pick(wv, lr, (j0 - col) & 31);
             const bool take = valid && ((word >> (lr & 31)) & 1u);
             const uint32_t tm = __ballot_sync(kFull, take);
             const int L = tm == kFull ? 32 : __ffs(~tm) - 1;    // rows t..t-L+1 are taken
-            const int pa = __shfl_sync(kFull, rllo, lr & 31), pb = __shfl_sync(kFull, rlhi, lr & 31);
-            const int sa = __shfl_sync(kFull, sklo, lr & 31), sb = __shfl_sync(kFull, skhi, lr & 31);
+            const int pos = pick(rlv, lr, lr & 31);
+            const int skr = pick(skv, lr, lr & 31);
             if (lane < L) {
-                const int pos = lr < 32 ? pa : pb;
                 if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
                 else chosen[(size_t)item * n + order[pos]] = 1;
             }
@@ -777,7 +781,7 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             }
             const int vL = __shfl_sync(kFull, (int)valid, L);
             const int colL = __shfl_sync(kFull, col, L);
-            const int skL = __shfl_sync(kFull, lr < 32 ? sa : sb, L);
+            const int skL = __shfl_sync(kFull, skr, L);
             j = colL;
             if (vL) {
                 t = skL;                                      // row t-L is skipped: next(i), -1 = past n
