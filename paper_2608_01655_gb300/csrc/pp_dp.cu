@@ -803,7 +803,12 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
 // values, and no kept row's value or bit changes.  With `cnt` the prefix
 // counts of positive profits in preorder, x has a positive strict descendant
 // iff cnt[next(x)] - cnt[x + 1] > 0, and row i is kept iff it is a root or its
-// parent has one.  Kept rows are listed in sweep order (decreasing i).
+// parent has one.  A kept row i that is itself an identity (p_i <= 0 and no
+// positive strict descendant: D[i] = D[next(i)] = the row just computed, all
+// bits "skip") and has no skip-row stack operation is dropped as well.  Kept
+// rows are listed in sweep order (decreasing i); every position records the
+// first kept row at or after it in preorder, so a skip to a dropped row lands
+// where the all-"skip" walk through it would.
 // ===========================================================================
 __device__ __forceinline__ int block_exclusive_scan(int v, int *total, int *sh)
 {
@@ -889,8 +894,14 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
             if (r < n) {
                 kp[v] = true;
                 if (prune) {
-                    const int2 sp = pspan[n - 1 - r];
+                    const int i = n - 1 - r;
+                    const int2 sp = pspan[i];
                     kp[v] = sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0;
+                    // an identity row (p <= 0 and no positive strict descendant, so
+                    // D[i] = D[next(i)] and every bit is "skip") without a stack
+                    // operation leaves the register state unchanged: drop it too
+                    if (kp[v] && (wmeta[i] & kWaveStackOps) == 0 && cnt[next[i]] - cnt[i + 1] == 0 && pval(i) <= 0)
+                        kp[v] = false;
                 }
             }
             kc += kp[v];
@@ -906,7 +917,7 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
                     kx[i] = ex++;
                     wmine += wpre[i];
                 } else {
-                    kx[i] = -1;
+                    kx[i] = ex - 1;         // the first kept row at or after position i (-1: none)
                 }
             }
         }
