@@ -1044,11 +1044,15 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     if (g_tune_cl > 0) cl_hi = std::min(g_tune_cl, 8);
     // Shape chosen by timing whole plans (paper-scale and source-dependent
     // workloads): the widest cluster the SMs per item allow, then columns per
-    // thread grown until a CTA has at most 4 warps (one per scheduler).
+    // thread grown until a CTA has at most 4 warps, but to at most 4 columns
+    // (8 columns per thread cost more than the extra warps).  At 16 items only
+    // 15 clusters of 8 find an SM per CTA on 152 SMs; the 16th shares SMs, and
+    // that still beats narrower clusters on the plan (not on a single launch).
     for (int CL = cl_hi; CL >= 1; --CL) {
         const int64_t cols = (k + CL - 1) / CL;
         int C = WMAX;
-        while ((cols + 32 * C - 1) / (32 * C) > 4 && C < 8) C *= 2;
+        while ((cols + 32 * C - 1) / (32 * C) > 4 && C < 4) C *= 2;
+        if ((cols + 32 * C - 1) / (32 * C) > 16) C = 8;
         if (g_tune_c > 0) C = std::max(std::min(g_tune_c, 8), WMAX);
         const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
         if (WPC > 16) continue;
