@@ -129,6 +129,13 @@ def oracle_update(inst, prob, rng):
     return inst.n * int(inst.budget[h]), time.perf_counter() - t0
 
 
+def _config(inst, S):
+    """The workload of both arms (the reference arm times the oracle on it)."""
+    return {"workload": inst.name, "n": inst.n, "W": inst.W, "k": int(inst.budget.max()), "starts": S,
+            "rounds": inst.rounds, "mode": "source-dependent" if inst.mode else "requester-side",
+            "l2": "flushed between steps (256 MiB write)", "parallelism": f"starts (weak, {S} per GPU)"}
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -155,9 +162,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * secs / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
-        "data": "synthetic", "config": {"workload": inst.name, "n": inst.n, "W": inst.W,
-                                        "k": int(inst.budget[0]), "starts": inst.starts,
-                                        "rounds": inst.rounds},
+        "data": "synthetic", "config": _config(inst, inst.starts),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "gpu_launches": 0,
@@ -450,9 +455,7 @@ def run_native(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": {"workload": inst.name, "n": n, "W": inst.W, "k": k, "starts": S, "rounds": R,
-                       "mode": "source-dependent", "l2": "flushed between steps (256 MiB write)",
-                       "parallelism": f"starts (weak, {S} per GPU)"},
+            "config": _config(inst, S),
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

@@ -249,6 +249,26 @@ def test_plan_top2_marginals(pp, oracle_lib):
                 _compare_plans(g, o)
 
 
+def test_plan_matches_oracle_digests(pp):
+    """Whole plans at the paper-scale and stress sizes against the oracle's own
+    plans, stored as digests by tests/golden/make_plan_digests.py (the oracle
+    needs minutes on many cores there): objective, returned candidate and the
+    SHA-256 of the placement identical."""
+    import hashlib
+    import os
+    path = os.path.join(os.path.dirname(__file__), "golden", "plan_digests.txt")
+    rows = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    assert rows
+    cfg_of = {c["name"]: k for k, c in wl.CONFIGS.items()}
+    for name, obj, best, digest in rows:
+        inst = wl.make(cfg_of[name])
+        with pp.Instance.from_workload(inst) as ppi:
+            g = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds)
+        assert g.objective == int(obj)
+        assert g.best_start == int(best)
+        assert hashlib.sha256(g.placement.astype(np.uint8).tobytes()).hexdigest() == digest
+
+
 def _shifted(rng, inst, kind):
     dem = inst.demand.copy()
     if kind == 0:
