@@ -672,6 +672,7 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 // (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
 // replaces bit h of the holder masks by the traced set.
 // ===========================================================================
+constexpr int kPruneCluster = 8;         // CTAs per item of the pruned-sweep kernel
 constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (a multiple of 32)
 
 __global__ void __launch_bounds__(256)
@@ -837,6 +838,40 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int *total, int *sh)
     return before + x - v;
 }
 
+// Exclusive scan over the CTAs of the cluster of one value per CTA (`v`, the
+// same in every thread of the CTA).  Returns this CTA's offset and the cluster
+// total.  The cluster barriers also order the global writes made before the
+// call against the reads of other CTAs after it.
+__device__ __forceinline__ int ld_dsmem_s32(uint32_t addr)
+{
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ int cluster_exclusive_scan(int v, int *total, int *slot, int *bcast)
+{
+    const int CLn = (int)cluster_nctarank(), cr = (int)cluster_ctarank();
+    if (threadIdx.x == 0) *slot = v;
+    cluster_sync_all();
+    if (threadIdx.x == 0) {
+        int ex = 0, tot = 0;
+        for (int c = 0; c < CLn; ++c) {
+            const int x = ld_dsmem_s32(map_to_rank(smem_addr(slot), (uint32_t)c));
+            ex += c < cr ? x : 0;
+            tot += x;
+        }
+        bcast[0] = ex;
+        bcast[1] = tot;
+    }
+    cluster_sync_all();           // every slot read: they may be written again
+    *total = bcast[1];
+    return bcast[0];
+}
+
+// One cluster of CL CTAs per item: every pass splits its index range into CL
+// contiguous slices, each CTA walks its slice in tiles of T*V elements (V per
+// thread, one block scan per tile), and the slices are joined by a scan over
+// the cluster's CTAs.
 template <bool BYNODE>
 __global__ void __launch_bounds__(1024)
 k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
@@ -845,92 +880,110 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         const int32_t *__restrict__ item_active, DpWork w, int prune,
         unsigned long long *__restrict__ rows_kept)
 {
-    // every pass walks tiles of T*V consecutive elements, V per thread, with one
-    // block scan per tile and a carry between tiles (all threads run every tile)
     constexpr int V = 4;
     __shared__ int sh[32];
-    const int item = blockIdx.x;
-    if (item_active && !item_active[item]) return;
+    __shared__ int slot, bcast[2];
+    const int CL = (int)cluster_nctarank(), cr = (int)cluster_ctarank();
+    const int item = blockIdx.x / CL;
+    if (item_active && !item_active[item]) return;       // uniform over the cluster
     const int64_t *Pp = profit + (size_t)item * n;
     int32_t *cnt = w.cnt + (size_t)item * (n + 1);
     int32_t *rl = w.rowlist + (size_t)item * n;
     int32_t *kx = w.kidx + (size_t)item * n;
     const int T = blockDim.x, t = threadIdx.x, tile = T * V;
     auto pval = [&](int i) { return Pp[BYNODE ? order[i] : i]; };
+    auto slice = [&](int len, int &lo, int &hi) {
+        const int per = (len + CL - 1) / CL;
+        lo = min(len, cr * per);
+        hi = min(len, lo + per);
+    };
+    int lo, hi, total;
 
     // prefix counts of positive profits, preorder
-    int carry = 0;
-    for (int base = 0; base < n; base += tile) {
-        int f[V], c = 0, total;
+    slice(n, lo, hi);
+    int mine = 0;
+    for (int i = lo + t; i < hi; i += T) mine += pval(i) > 0;
+    block_exclusive_scan(mine, &total, sh);
+    int carry = cluster_exclusive_scan(total, &total, &slot, bcast);
+    const int npos = total;
+    for (int base = lo; base < hi; base += tile) {
+        int f[V], c = 0;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int i = base + t * V + v;
-            f[v] = i < n && pval(i) > 0;
+            f[v] = i < hi && pval(i) > 0;
             c += f[v];
         }
-        int ex = block_exclusive_scan(c, &total, sh) + carry;
+        int tt;
+        int ex = block_exclusive_scan(c, &tt, sh) + carry;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int i = base + t * V + v;
-            if (i < n) {
+            if (i < hi) {
                 cnt[i] = ex;
                 ex += f[v];
             }
         }
-        carry += total;
+        carry += tt;
     }
-    if (t == 0) cnt[n] = carry;
-    __syncthreads();
+    if (cr == 0 && t == 0) cnt[n] = npos;
+    cluster_sync_all();                                   // cnt complete for every CTA
 
     // kept rows in sweep order r = n - 1 - i, their kept index, their total weight
-    int kcarry = 0, wmine = 0;
-    for (int base = 0; base < n; base += tile) {
+    auto keep = [&](int r) -> bool {
+        if (!prune) return true;
+        const int i = n - 1 - r;
+        const int2 sp = pspan[i];
+        if (!(sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0)) return false;
+        // an identity row (p <= 0 and no positive strict descendant, so D[i] =
+        // D[next(i)] and every bit is "skip") without a stack operation leaves
+        // the register state unchanged: drop it too
+        return !((wmeta[i] & kWaveStackOps) == 0 && cnt[next[i]] - cnt[i + 1] == 0 && pval(i) <= 0);
+    };
+    slice(n, lo, hi);
+    int kmine = 0, wmine = 0;
+    for (int r = lo + t; r < hi; r += T)
+        if (keep(r)) {
+            kmine += 1;
+            wmine += wpre[n - 1 - r];
+        }
+    block_exclusive_scan(kmine, &total, sh);
+    int kcarry = cluster_exclusive_scan(total, &total, &slot, bcast);
+    const int nk = total;
+    block_exclusive_scan(wmine, &total, sh);
+    int wtot;
+    cluster_exclusive_scan(total, &wtot, &slot, bcast);   // weight of all kept rows
+    for (int base = lo; base < hi; base += tile) {
         bool kp[V];
-        int kc = 0, total;
+        int kc = 0;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int r = base + t * V + v;
-            kp[v] = false;
-            if (r < n) {
-                kp[v] = true;
-                if (prune) {
-                    const int i = n - 1 - r;
-                    const int2 sp = pspan[i];
-                    kp[v] = sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0;
-                    // an identity row (p <= 0 and no positive strict descendant, so
-                    // D[i] = D[next(i)] and every bit is "skip") without a stack
-                    // operation leaves the register state unchanged: drop it too
-                    if (kp[v] && (wmeta[i] & kWaveStackOps) == 0 && cnt[next[i]] - cnt[i + 1] == 0 && pval(i) <= 0)
-                        kp[v] = false;
-                }
-            }
+            kp[v] = r < hi && keep(r);
             kc += kp[v];
         }
-        int ex = block_exclusive_scan(kc, &total, sh) + kcarry;
+        int tt;
+        int ex = block_exclusive_scan(kc, &tt, sh) + kcarry;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int r = base + t * V + v;
-            if (r < n) {
+            if (r < hi) {
                 const int i = n - 1 - r;
                 if (kp[v]) {
                     rl[ex] = i;
                     kx[i] = ex++;
-                    wmine += wpre[i];
                 } else {
                     kx[i] = ex - 1;         // the first kept row at or after position i (-1: none)
                 }
             }
         }
-        kcarry += total;
+        kcarry += tt;
     }
-    const int nk = kcarry;
-    int wtot;
-    block_exclusive_scan(wmine, &wtot, sh);                // weight of all kept rows
-    if (t == 0) {
+    if (cr == 0 && t == 0) {
         w.nkept[item] = nk;
         if (rows_kept) atomicAdd(rows_kept, (unsigned long long)nk);
     }
-    __syncthreads();
+    cluster_sync_all();                                   // rl and kx complete
 
     // per kept row: skip target, the DP's row stream (profit, metadata) and
     // the suffix weights of the traceback
@@ -938,14 +991,18 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
     int32_t *ws = w.wsuf + (size_t)item * (n + 1);
     int64_t *rp = w.rowp + (size_t)item * n;
     int32_t *rm = w.rowm + (size_t)item * n;
-    int wcarry = 0;
-    for (int base = 0; base < nk; base += tile) {
-        int wq[V], wl = 0, total;
+    slice(nk, lo, hi);
+    wmine = 0;
+    for (int q = lo + t; q < hi; q += T) wmine += wpre[rl[q]];
+    block_exclusive_scan(wmine, &total, sh);
+    int wcarry = cluster_exclusive_scan(total, &total, &slot, bcast);
+    for (int base = lo; base < hi; base += tile) {
+        int wq[V], wl = 0;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int q = base + t * V + v;
             wq[v] = 0;
-            if (q < nk) {
+            if (q < hi) {
                 const int i = rl[q];
                 const int nx = next[i];
                 sk[q] = nx < n ? kx[nx] : -1;
@@ -955,20 +1012,21 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
             }
             wl += wq[v];
         }
-        int ex = block_exclusive_scan(wl, &total, sh) + wcarry;   // weight of kept rows before q
+        int tt;
+        int ex = block_exclusive_scan(wl, &tt, sh) + wcarry;   // weight of kept rows before q
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int q = base + t * V + v;
-            if (q < nk) {
+            if (q < hi) {
                 ws[q] = wtot - ex;                                 // weight of kept rows q..nk-1
                 ex += wq[v];
             }
         }
-        wcarry += total;
+        wcarry += tt;
     }
-    if (t == 0) ws[nk] = 0;
-    __syncthreads();
-    for (int q = t; q < nk; q += T) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
+    if (cr == 0 && t == 0) ws[nk] = 0;
+    cluster_sync_all();                                   // sk complete
+    for (int q = lo + t; q < hi; q += T) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
 }
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1158,14 +1216,28 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
                                    unsigned long long *rows_kept)
 {
     // the pruned sweep of every item, then the DP over its kept rows
-    if (by_node)
-        k_prune<true><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
-                                              inst->d_wpre, inst->d_wave, item_active, work, !g_tune_noprune,
-                                              rows_kept);
-    else
-        k_prune<false><<<batch, 1024, 0, st>>>(inst->n, profit, inst->d_order, inst->d_next, inst->d_pspan,
-                                               inst->d_wpre, inst->d_wave, item_active, work, !g_tune_noprune,
-                                               rows_kept);
+    {
+        cudaLaunchConfig_t pc = {};
+        pc.gridDim = dim3(kPruneCluster * batch);
+        pc.blockDim = dim3(1024);
+        pc.stream = st;
+        cudaLaunchAttribute pa[1];
+        pa[0].id = cudaLaunchAttributeClusterDimension;
+        pa[0].val.clusterDim.x = kPruneCluster;
+        pa[0].val.clusterDim.y = 1;
+        pa[0].val.clusterDim.z = 1;
+        pc.attrs = pa;
+        pc.numAttrs = 1;
+        const int32_t *ord = inst->d_order, *nxt = inst->d_next, *wp = inst->d_wpre, *wm = inst->d_wave;
+        const int2 *psp = inst->d_pspan;
+        const int pr = !g_tune_noprune;
+        if (by_node)
+            PP_CUDA(cudaLaunchKernelEx(&pc, k_prune<true>, inst->n, profit, ord, nxt, psp, wp, wm, item_active,
+                                       work, pr, rows_kept));
+        else
+            PP_CUDA(cudaLaunchKernelEx(&pc, k_prune<false>, inst->n, profit, ord, nxt, psp, wp, wm, item_active,
+                                       work, pr, rows_kept));
+    }
     PP_CUDA(cudaGetLastError());
     uint32_t *bits = work.bits;
     const int32_t *nkept = work.nkept;
