@@ -395,7 +395,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
 #pragma unroll
             for (int u = 0; u < kSub; ++u) pv[u] = my_p[s8 + u];
             // one row of Eq. 9 for this warp's columns; STACK: the row may push or pop
-            auto row = [&](const int u, const bool STACK) {
+            auto row = [&](const int u, const bool STACK, const int SRC) {
                 const int64_t p = pv[u];
                 // bnd[q] = D[i+1][base - WMAX + 1 + q]: row r-1 of the previous warp
                 // (the first warp's sv is all zero: column 0 of every row is 0)
@@ -419,7 +419,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                 const bool from_cur = (cb >> u) & 1u;
 #pragma unroll
                 for (int c = 0; c < C; ++c) {
-                    const int64_t sk = from_cur ? cur[c] : top[c];
+                    const int64_t sk = SRC == 1 ? cur[c] : SRC == 2 ? top[c] : (from_cur ? cur[c] : top[c]);
                     const int64_t t = p + sh[c];
                     const bool take = t > sk;
                     cur[c] = take ? t : sk;
@@ -459,12 +459,18 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                     }
                 }
             };
+            const uint32_t cb8 = cb & ((1u << kSub) - 1);
             if (stk8 == 0) {
+                if (cb8 == 0) {
 #pragma unroll
-                for (int u = 0; u < kSub; ++u) row(u, false);       // no push or pop in these rows
+                    for (int u = 0; u < kSub; ++u) row(u, false, 2);   // every skip row is the top
+                } else {
+#pragma unroll
+                    for (int u = 0; u < kSub; ++u) row(u, false, 0);   // no push or pop in these rows
+                }
             } else {
 #pragma unroll
-                for (int u = 0; u < kSub; ++u) row(u, true);
+                for (int u = 0; u < kSub; ++u) row(u, true, 0);
             }
 #pragma unroll
             for (int c = 0; c < C; ++c) wbits[c] |= wb8[c] << s8;
