@@ -399,6 +399,33 @@ def test_degenerate_instances(pp, oracle_lib):
             _compare_plans(g, o)
 
 
+def test_degenerate_safeguards_and_epoch_updates(pp, oracle_lib):
+    """Requester-side n = 0, all budgets 0, one worker and one chunk: safeguard
+    candidates, plans with them and epoch updates agree with the oracle."""
+    for n, W, k in [(0, 2, 5), (1, 1, 1), (6, 3, 0), (1, 32, 3), (4, 1, 2)]:
+        rng = np.random.default_rng(n * 7 + W)
+        inst = wl.random_small(rng, n, W, 0, k_max=max(k, 1)) if n else wl.Instance(
+            "empty", 0, W, np.zeros(0, np.int32), np.zeros(0, np.int32), np.zeros((W, 0), np.int64),
+            np.zeros((W, 0), np.int64), np.zeros((W, 0), np.int64), 0, np.full(W, k, np.int32), 1, 1)
+        if k == 0:
+            inst.budget[:] = 0
+        prob = oracle_lib.Problem.from_instance(inst)
+        old = np.zeros((W, n), np.uint8)
+        with pp.Instance.from_workload(inst) as ppi:
+            gpl, gobj = pp.pp_safeguards(ppi)
+            g = pp.pp_plan_run(ppi, 2, None, 2)
+            r = pp.pp_replan(ppi, old, 2, 2, 30000, 30000)
+        opl, oobj = oracle_lib.safeguards(prob)
+        np.testing.assert_array_equal(gpl, opl)
+        np.testing.assert_array_equal(gobj, oobj)
+        _compare_plans(g, oracle_lib.plan(prob, 2, 2))
+        o = oracle_lib.replan(prob, old, 2, 2, 30000, 30000)
+        assert (r.incumbent_objective, r.new_objective, r.materialization_cost, r.break_even_requests,
+                r.adopted) == (o.incumbent_objective, o.new_objective, o.materialization_cost,
+                               o.break_even_requests, o.adopted)
+        np.testing.assert_array_equal(r.placement, o.placement)
+
+
 def test_device_bounds_errors(pp):
     """A budget above the declared bound and a worker id out of range are
     reported through the status word, not by faulting."""
