@@ -331,6 +331,9 @@ def run_native(args):
         from paper_2608_01655_gb300 import shard
         all_orders = pp.pp_default_orders(ppi, S * world)
         orders = all_orders[shard.my_starts(S * world, rank, world)]
+    # the requester-side safeguards are candidates of the whole plan, not of a
+    # start: with several ranks only the starts are sharded and compared
+    sg = world == 1
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")   # 2x the 129 MB L2
 
     def barrier():
@@ -339,7 +342,7 @@ def run_native(args):
 
     res = None
     for _ in range(args.warmup):
-        res = pp.pp_plan_run(ppi, S, orders, R)
+        res = pp.pp_plan_run(ppi, S, orders, R, safeguards=sg)
     cells_per_plan = res.dp_cells
     launches_per_plan = res.kernel_launches
     times, phase_sum = [], [0.0, 0.0, 0.0]
@@ -352,7 +355,7 @@ def run_native(args):
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             # events around every launch of the plan (read after the plan returns)
-            res = pp.pp_plan_run(ppi, S, orders, R, time_phases=True)
+            res = pp.pp_plan_run(ppi, S, orders, R, time_phases=True, safeguards=sg)
             e1.record(stream)
             torch.cuda.synchronize()
             barrier()
@@ -421,7 +424,7 @@ def run_native(args):
         t0 = time.perf_counter()
         with pp.Instance(host["parent"], host["weight"], host["demand"], host["recompute"],
                          host["transfer"], inst.mode, host["budget"]) as ppe:
-            r2 = pp.pp_plan_run(ppe, S, orders, R)
+            r2 = pp.pp_plan_run(ppe, S, orders, R, safeguards=sg)
         torch.cuda.synchronize()
         if it >= args.warmup:
             e2e_times.append(time.perf_counter() - t0)
