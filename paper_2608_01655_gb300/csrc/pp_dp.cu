@@ -188,27 +188,27 @@ template <int C, int WMAX>
 __device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t (&bnd)[WMAX], bool lane,
                                           int w, int64_t (&sh)[C])
 {
-    if (WMAX == 1) {
+    if constexpr (WMAX == 1) {
         shift_by<C, WMAX, 1>(cur, bnd, lane, sh);
-        return;
-    }
-    // branch-free: every candidate shift, then a select by w (a per-row branch
-    // would end the unrolled straight-line block of rows)
-    int64_t up[WMAX];      // up[q]: column C-1-q of the lane to the left (lane 0: the boundary)
+    } else {
+        // branch-free: every candidate shift, then a select by w (a per-row
+        // branch would end the unrolled straight-line block of rows)
+        int64_t up[WMAX];  // up[q]: column C-1-q of the lane to the left (lane 0: the boundary)
 #pragma unroll
-    for (int q = 0; q < WMAX; ++q) {
-        const int64_t v = __shfl_up_sync(kFull, cur[C - 1 - q], 1);
-        up[q] = lane ? bnd[WMAX - 1 - q] : v;
-    }
-#pragma unroll
-    for (int c = 0; c < C; ++c) {
-        int64_t v = c >= 1 ? cur[c - 1 < 0 ? 0 : c - 1] : up[0];
-#pragma unroll
-        for (int ww = 2; ww <= WMAX; ++ww) {
-            const int64_t cand = c >= ww ? cur[c - ww < 0 ? 0 : c - ww] : up[ww - 1 - c < 0 ? 0 : ww - 1 - c];
-            v = w == ww ? cand : v;
+        for (int q = 0; q < WMAX; ++q) {
+            const int64_t v = __shfl_up_sync(kFull, cur[C - 1 - q], 1);
+            up[q] = lane ? bnd[WMAX - 1 - q] : v;
         }
-        sh[c] = v;
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+            int64_t v = c >= 1 ? cur[c - 1 < 0 ? 0 : c - 1] : up[0];
+#pragma unroll
+            for (int ww = 2; ww <= WMAX; ++ww) {
+                const int64_t cand = c >= ww ? cur[c - ww < 0 ? 0 : c - ww] : up[ww - 1 - c < 0 ? 0 : ww - 1 - c];
+                v = w == ww ? cand : v;
+            }
+            sh[c] = v;
+        }
     }
 }
 
