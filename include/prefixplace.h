@@ -56,7 +56,8 @@ typedef enum {
 
 enum { PP_TRANSFER_REQUESTER = 0, PP_TRANSFER_SOURCE = 1 };
 
-/* Optional outputs of pp_plan_run.  Array members may be NULL. */
+/* Optional inputs and outputs of pp_plan_run / pp_replan.  Zero-initialise it:
+ * every "in" field's zero is the default.  Array members may be NULL. */
 typedef struct {
     int64_t *per_start_objective;  /* [n_starts] host, out: objective of each candidate */
     int32_t *per_start_sweeps;     /* [n_starts] host, out: refinement sweeps run */
