@@ -317,6 +317,20 @@ pp_status pp_test_inject(int32_t kind, int32_t value);
 pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_budget, int32_t *out);
 
 /*
+ * pp_dp_split -- whether pp_tree_dp runs `batch` items with budgets up to
+ * `max_budget` as two concurrent launches (host out[5]): items of the wide
+ * launch (0 = one launch; its shape is that of pp_dp_geometry), CTAs per
+ * cluster and warps per CTA of the narrow launch that takes the other items
+ * (the ones with the fewest kept rows), its skip-row stack levels in shared
+ * memory, and the wide launch's shared memory bytes per CTA.  A split is
+ * used when the batch exceeds, by at most 2, the number of the wide clusters
+ * that the device holds at one CTA per SM (15 clusters of 8 CTAs on a
+ * 152-SM GB300); results and decision bits do not depend on it.
+ * Errors: PP_EINVAL.
+ */
+pp_status pp_dp_split(const pp_instance *inst, int32_t batch, int32_t max_budget, int32_t *out);
+
+/*
  * pp_tune_dp -- process-wide override of the DP launch shape, for tuning
  * sweeps: CTAs per cluster (1..8, 0 = automatic), columns per thread (power
  * of two up to 16, 0 = automatic), force_flat != 0 selects the one-CTA kernel,

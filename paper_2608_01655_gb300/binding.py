@@ -62,6 +62,7 @@ _SIGS = {
     "pp_plan_run": [_P, _i32, _P, _i32, _P, _P, ctypes.POINTER(PlanStats), _P],
     "pp_test_inject": [_i32, _i32],
     "pp_dp_geometry": [_P, _i32, _i32, _P],
+    "pp_dp_split": [_P, _i32, _i32, _P],
     "pp_tune_dp": [_i32, _i32, _i32, _i32],
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
     "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
@@ -287,6 +288,14 @@ def pp_dp_geometry(inst: Instance, batch: int, max_budget: int) -> dict:
     _check(_lib.pp_dp_geometry(inst.handle, int(batch), int(max_budget), _host(out)))
     keys = ["wave", "cluster_ctas", "warps_per_cta", "columns_per_thread", "warps_per_dp",
             "stack_levels_smem", "smem_bytes", "kpad"]
+    return {k: int(v) for k, v in zip(keys, out)}
+
+
+def pp_dp_split(inst: Instance, batch: int, max_budget: int) -> dict:
+    out = np.zeros(5, np.int32)
+    _check(_lib.pp_dp_split(inst.handle, int(batch), int(max_budget), _host(out)))
+    keys = ["wide_items", "narrow_cluster_ctas", "narrow_warps_per_cta", "narrow_stack_levels_smem",
+            "wide_smem_bytes"]
     return {k: int(v) for k, v in zip(keys, out)}
 
 

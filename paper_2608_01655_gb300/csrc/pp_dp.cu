@@ -234,13 +234,34 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                const int32_t *__restrict__ item_budget, int32_t max_budget,
                const int32_t *__restrict__ item_active, int64_t *__restrict__ best,
                uint32_t *__restrict__ bits, int64_t *__restrict__ gstack, int L_smem, int L_glob,
-               int32_t *__restrict__ status)
+               int32_t *__restrict__ status, int32_t batch, int32_t slot_base, int32_t ranked)
 {
     using namespace wavecfg;
     extern __shared__ __align__(16) unsigned char smem[];
     const int CL = (int)cluster_nctarank();
     const int cr = (int)cluster_ctarank();
-    const int item = blockIdx.x / CL;
+    int item = blockIdx.x / CL;
+    if (ranked) {
+        // split launch (batch <= 32): slot s of the two launches takes the
+        // item of rank s by kept rows, most first (ties to the lower index,
+        // inactive items last), so the narrower second launch gets the
+        // smallest sweeps; every CTA of a cluster computes the same item
+        __shared__ int s_item;
+        if (threadIdx.x < 32) {
+            const int x = threadIdx.x;
+            const int key = x < batch && (!item_active || item_active[x]) ? nkept[x] : -1;
+            int rank = 0;
+            for (int y = 0; y < batch; ++y) {
+                const int ky = __shfl_sync(kFull, key, y);
+                rank += ky > key || (ky == key && y < x);
+            }
+            const unsigned m = __ballot_sync(kFull, x < batch && rank == slot_base + item);
+            if (x == 0) s_item = m ? __ffs((int)m) - 1 : -1;
+        }
+        __syncthreads();
+        item = s_item;
+        if (item < 0) return;           // no such slot: uniform over the cluster
+    }
     const int NT = blockDim.x;
     const int WPC = NT >> 5;
     const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -263,7 +284,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
     uint64_t *ring = reinterpret_cast<uint64_t *>(smem);                           // [WPC][kRing][WMAX]
     int4 *mstage = reinterpret_cast<int4 *>(ring + (size_t)WPC * kRing * WMAX);    // [WPC][32] (p, m)
     uint32_t *ack = reinterpret_cast<uint32_t *>(mstage + (size_t)WPC * 32);       // [WPC]
-    int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX)); // [L_smem][C][NT]
+    int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX)); // [WPC][L_smem][C][32]
     for (int x = threadIdx.x; x < WPC * kRing * WMAX; x += NT) ring[x] = kLapBit;  // lap of row -1
     if (threadIdx.x < WPC) ack[threadIdx.x] = 0;
     cluster_sync_all();     // every CTA initialised before any remote write
@@ -289,6 +310,9 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
     uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
     int64_t *const my_gst = gst + threadIdx.x;
+    // this warp's shared-memory stack levels: a column's word of a level sits
+    // at a compile-time offset from the lane's base
+    int64_t *const my_stk = stk + (size_t)wl * L_smem * C * 32 + lane;
     // the kept rows of the pruned sweep, with their profit and metadata
     // gathered in sweep order
     const int nrows = nkept[item];
@@ -448,7 +472,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                         for (int c = 0; c < C; ++c) top[c] = cur[c];
                         if (lvl < L_smem) {
 #pragma unroll
-                            for (int c = 0; c < C; ++c) stk[((size_t)lvl * C + c) * NT + threadIdx.x] = cur[c];
+                            for (int c = 0; c < C; ++c) my_stk[((size_t)lvl * C + c) * 32] = cur[c];
                         } else {
 #pragma unroll
                             for (int c = 0; c < C; ++c) my_gst[(size_t)(lvl - L_smem) * CL * C * NT + (size_t)c * NT] = cur[c];
@@ -457,7 +481,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                         const int lvl = my_lv[s8 + u];
                         if (lvl < L_smem) {
 #pragma unroll
-                            for (int c = 0; c < C; ++c) top[c] = stk[((size_t)lvl * C + c) * NT + threadIdx.x];
+                            for (int c = 0; c < C; ++c) top[c] = my_stk[((size_t)lvl * C + c) * 32];
                         } else {
 #pragma unroll
                             for (int c = 0; c < C; ++c) top[c] = my_gst[(size_t)(lvl - L_smem) * CL * C * NT + (size_t)c * NT];
@@ -1002,7 +1026,7 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
 
     // per kept row: skip target, the DP's row stream (profit, metadata) and
     // the suffix weights of the traceback
-    int32_t *sk = w.skip + (size_t)item * n, *sk2 = w.skip2 + (size_t)item * n;
+    int32_t *sk = w.skip + (size_t)item * n;
     int32_t *ws = w.wsuf + (size_t)item * (n + 1);
     int64_t *rp = w.rowp + (size_t)item * n;
     int32_t *rm = w.rowm + (size_t)item * n;
@@ -1040,8 +1064,6 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         wcarry += tt;
     }
     if (cr == 0 && t == 0) ws[nk] = 0;
-    cluster_sync_all();                                   // sk complete
-    for (int q = lo + t; q < hi; q += T) sk2[q] = sk[q] < 0 ? -1 : sk[sk[q]];
 }
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1049,7 +1071,7 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 size_t dp_work_bytes(int batch, int n, int words)
 {
     const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
-    return align256(B * nb * words * 4) + 5 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
+    return align256(B * nb * words * 4) + 4 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
            align256(B * 4) + align256(B * N * 8);
 }
 
@@ -1069,8 +1091,6 @@ DpWork dp_work_split(void *base, int batch, int n, int words)
     w.nkept = reinterpret_cast<int32_t *>(p);
     p += align256(B * 4);
     w.skip = reinterpret_cast<int32_t *>(p);
-    p += align256(B * N * 4);
-    w.skip2 = reinterpret_cast<int32_t *>(p);
     p += align256(B * N * 4);
     w.wsuf = reinterpret_cast<int32_t *>(p);
     p += align256(B * (N + 1) * 4);
@@ -1106,6 +1126,69 @@ static int max_smem_optin(const pp_instance *inst)
 // Geometry overrides set by pp_tune_dp (0 = automatic).
 static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0, g_tune_noprune = 0;
 
+// Split launch: measured on GB300 (152 SMs), the placement of clusters of 8
+// CTAs at one CTA per SM finds room for 15 of them; a 16th cluster then shares
+// SMs with other items and slows them and itself by ~25% per row.  When the
+// batch exceeds that count by at most 2, the extra items (the smallest
+// sweeps, by rank in the kernel) run as clusters of CL / 2 CTAs on the SMs
+// that are left, in a second launch on its own stream.
+static void split_geometry(const pp_instance *inst, int batch, const void *fn, const cudaLaunchConfig_t &cfg0,
+                           int smem_max, DpGeom *g)
+{
+    if (g_tune_cl > 0 || g_tune_c > 0 || batch < 2 || batch > 32 || g->CL < 2 || (g->CL & 1) || 2 * g->WPC > 16)
+        return;
+    int per_sm = 0;
+    cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, inst->device);
+    const size_t excl = std::max(g->smem, (size_t)per_sm / 2);   // two CTAs never fit in one SM
+    if (excl > (size_t)smem_max) return;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)excl) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    cudaLaunchConfig_t cfg = cfg0;
+    cfg.dynamicSmemBytes = excl;
+    int m1 = 0;
+    if (cudaOccupancyMaxActiveClusters(&m1, fn, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    if (m1 < 1 || batch <= m1 || batch - m1 > 2) return;
+    const int CL2 = g->CL / 2, WPC2 = 2 * g->WPC;
+    const size_t fixed2 = wave_fixed_bytes(WPC2, g->WMAX);
+    const size_t level2 = (size_t)g->C * WPC2 * 32 * sizeof(int64_t);
+    if (fixed2 > (size_t)smem_max) return;
+    const int L2 = (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed2) / level2);
+    const size_t smem2 = std::max(fixed2 + (size_t)L2 * level2, excl);
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)std::max(excl, smem2)) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    cudaLaunchConfig_t cfg2 = cfg0;
+    cfg2.gridDim = dim3(CL2 * (batch - m1));
+    cfg2.blockDim = dim3(WPC2 * 32);
+    cfg2.dynamicSmemBytes = smem2;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg2.attrs = attr;
+    cfg2.numAttrs = 1;
+    int m2 = 0;
+    if (cudaOccupancyMaxActiveClusters(&m2, fn, &cfg2) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    if (m2 < batch - m1) return;
+    g->split = m1;
+    g->smem_x = excl;
+    g->CL2 = CL2;
+    g->WPC2 = WPC2;
+    g->L_smem2 = L2;
+    g->smem2 = smem2;
+}
+
 static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom *g)
 {
     const int WMAX = inst->max_weight <= 1 ? 1 : (inst->max_weight <= 2 ? 2 : 4);
@@ -1118,9 +1201,9 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     // Shape chosen by timing whole plans (paper-scale and source-dependent
     // workloads): the widest cluster the SMs per item allow, then columns per
     // thread grown until a CTA has at most 4 warps, but to at most 4 columns
-    // (8 columns per thread cost more than the extra warps).  At 16 items only
-    // 15 clusters of 8 find an SM per CTA on 152 SMs; the 16th shares SMs, and
-    // that still beats narrower clusters on the plan (not on a single launch).
+    // (8 columns per thread cost more than the extra warps).  A batch just
+    // above the number of such clusters that fit at one CTA per SM is split
+    // (split_geometry).
     for (int CL = cl_hi; CL >= 1; --CL) {
         const int64_t cols = (k + CL - 1) / CL;
         int C = WMAX;
@@ -1169,6 +1252,8 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
         g->words = g->kpad / 32;
         g->L_smem = L_smem;
         g->smem = smem;
+        g->split = 0;
+        split_geometry(inst, batch, fn, cfg, smem_max, g);
         return true;
     }
     return false;
@@ -1202,6 +1287,19 @@ bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int bat
     g->L_smem = inst->n > 0 ? (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed) / row_bytes) : 0;
     g->smem = fixed + (size_t)g->L_smem * row_bytes;
     return true;
+}
+
+static pp_status ensure_split_streams(pp_instance *inst)
+{
+    if (inst->split_hi) return PP_OK;
+    int least = 0, greatest = 0;
+    PP_CUDA(cudaDeviceGetStreamPriorityRange(&least, &greatest));
+    PP_CUDA(cudaStreamCreateWithPriority(&inst->split_hi, cudaStreamNonBlocking, greatest));
+    PP_CUDA(cudaStreamCreateWithPriority(&inst->split_lo, cudaStreamNonBlocking, least));
+    PP_CUDA(cudaEventCreateWithFlags(&inst->split_fork, cudaEventDisableTiming));
+    PP_CUDA(cudaEventCreateWithFlags(&inst->split_join_hi, cudaEventDisableTiming));
+    PP_CUDA(cudaEventCreateWithFlags(&inst->split_join_lo, cudaEventDisableTiming));
+    return PP_OK;
 }
 
 template <int C>
@@ -1259,28 +1357,49 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
     if (g.wave) {
         const void *fn = wave_kernel_for(g.C, g.WMAX);
         if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
-        PP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem));
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(g.CL * batch);
-        cfg.blockDim = dim3(g.WPC * 32);
-        cfg.dynamicSmemBytes = g.smem;
-        cfg.stream = st;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = g.CL;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        PP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)(g.split ? std::max(g.smem_x, g.smem2) : g.smem)));
         int32_t n = inst->n;
         int32_t nblk = (n + 31) / 32;
         const int64_t *rowp = work.rowp;
         const int32_t *rowm = work.rowm;
-        int32_t L_smem = g.L_smem, Lg = L_glob;
         int32_t *status = inst->d_status;
-        void *args[] = {&n, &nblk, (void *)&rowp, (void *)&rowm, (void *)&nkept, (void *)&item_budget, &max_budget,
-                        (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status};
-        PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
+        int32_t nb = batch;
+        auto launch = [&](int CL, int WPC, size_t smem, int32_t L_smem, int items, int32_t slot_base,
+                          cudaStream_t s) -> pp_status {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(CL * items);
+            cfg.blockDim = dim3(WPC * 32);
+            cfg.dynamicSmemBytes = smem;
+            cfg.stream = s;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = CL;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            int32_t Lg = L_glob, ranked = g.split > 0;
+            void *args[] = {&n, &nblk, (void *)&rowp, (void *)&rowm, (void *)&nkept, (void *)&item_budget,
+                            &max_budget, (void *)&item_active, &best, &bits, &gstack, &L_smem, &Lg, &status,
+                            &nb, &slot_base, &ranked};
+            PP_CUDA(cudaLaunchKernelExC(&cfg, fn, args));
+            return PP_OK;
+        };
+        if (!g.split) return launch(g.CL, g.WPC, g.smem, g.L_smem, batch, 0, st);
+        pp_status s;
+        if ((s = ensure_split_streams(inst))) return s;
+        // fork: the wide launch first, on the higher-priority stream, so its
+        // clusters are placed before the narrow ones take the SMs left over
+        PP_CUDA(cudaEventRecord(inst->split_fork, st));
+        PP_CUDA(cudaStreamWaitEvent(inst->split_hi, inst->split_fork, 0));
+        PP_CUDA(cudaStreamWaitEvent(inst->split_lo, inst->split_fork, 0));
+        if ((s = launch(g.CL, g.WPC, g.smem_x, g.L_smem, g.split, 0, inst->split_hi))) return s;
+        if ((s = launch(g.CL2, g.WPC2, g.smem2, g.L_smem2, batch - g.split, g.split, inst->split_lo))) return s;
+        PP_CUDA(cudaEventRecord(inst->split_join_hi, inst->split_hi));
+        PP_CUDA(cudaEventRecord(inst->split_join_lo, inst->split_lo));
+        PP_CUDA(cudaStreamWaitEvent(st, inst->split_join_hi, 0));
+        PP_CUDA(cudaStreamWaitEvent(st, inst->split_join_lo, 0));
         return PP_OK;
     }
     switch (g.C) {
@@ -1294,6 +1413,13 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
     }
 }
 
+// Skip-row stack levels below shared memory, per item (the larger need of the
+// two launches of a split).
+static int dp_global_levels(const pp_instance *inst, const DpGeom &g)
+{
+    return std::max(0, inst->stack_depth - (g.split ? std::min(g.L_smem, g.L_smem2) : g.L_smem));
+}
+
 pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
                          const int32_t *item_budget, const int32_t *item_active, const DpGeom &g,
                          int64_t *best, const DpWork &work, cudaStream_t st, int32_t max_budget,
@@ -1304,7 +1430,7 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
         PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
         return PP_OK;
     }
-    const int L_glob = inst->stack_depth - g.L_smem;
+    const int L_glob = dp_global_levels(inst, g);
     if (L_glob > 0) {
         pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
         if (s != PP_OK) return s;
@@ -1403,6 +1529,19 @@ extern "C" pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int3
     return PP_OK;
 }
 
+extern "C" pp_status pp_dp_split(const pp_instance *inst, int32_t batch, int32_t max_budget, int32_t *out)
+{
+    if (!inst || !out) return fail(PP_EINVAL, "null pointer");
+    DpGeom g;
+    if (!dp_geometry(inst, max_budget, &g, std::max(batch, 1))) return fail(PP_EINVAL, "max_budget out of range");
+    out[0] = g.split;
+    out[1] = g.split ? g.CL2 : 0;
+    out[2] = g.split ? g.WPC2 : 0;
+    out[3] = g.split ? g.L_smem2 : 0;
+    out[4] = g.split ? (int32_t)g.smem_x : 0;
+    return PP_OK;
+}
+
 // ===========================================================================
 // pp_tree_dp_noalloc: the same DP launch with the skip-row stack levels that do
 // not fit in shared memory kept in a fixed array of this library's device
@@ -1457,8 +1596,9 @@ extern "C" pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const 
         PP_CUDA(cudaMemsetAsync(best, 0, sizeof(int64_t) * batch, st));
         return PP_OK;
     }
-    const int L_glob = inst->stack_depth - g.L_smem;
-    const size_t need = (size_t)batch * (size_t)std::max(L_glob, 0) * (size_t)g.kpad * sizeof(int64_t);
+    g.split = 0;                        // one launch: no internal streams or events
+    const int L_glob = dp_global_levels(inst, g);
+    const size_t need = (size_t)batch * (size_t)L_glob * (size_t)g.kpad * sizeof(int64_t);
     if (need > kStaticStackBytes)
         return fail(PP_EINVAL, "pp_tree_dp_noalloc: this launch needs " + std::to_string(need) +
                                    " bytes of skip-row stack scratch, more than its fixed " +

@@ -234,6 +234,11 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     free_scratch(inst->sg);
     free_scratch(inst->rp);
     free_scratch(inst->top2);
+    if (inst->split_hi) cudaStreamDestroy(inst->split_hi);
+    if (inst->split_lo) cudaStreamDestroy(inst->split_lo);
+    if (inst->split_fork) cudaEventDestroy(inst->split_fork);
+    if (inst->split_join_hi) cudaEventDestroy(inst->split_join_hi);
+    if (inst->split_join_lo) cudaEventDestroy(inst->split_join_lo);
     cudaSetDevice(cur);
     delete inst;
     return PP_OK;

@@ -66,6 +66,16 @@ struct DpGeom {
     int WMAX = 1;     // largest chunk weight the wavefront kernel is built for
     int L_smem = 0;   // skip-row stack levels held in shared memory
     size_t smem = 0;  // dynamic shared memory per CTA
+    // Split launch (wavefront kernel, batch just above what clusters of CL
+    // CTAs hold at one CTA per SM): the `split` items with the most kept rows
+    // run as clusters of CL, the rest concurrently as clusters of CL2 = CL / 2
+    // CTAs x WPC2 = 2 * WPC warps on the SMs left over (same P, C and bit
+    // layout).  Both launches reserve more than half an SM's shared memory so
+    // that no SM hosts two CTAs.  split = 0: one launch.
+    int split = 0;
+    size_t smem_x = 0;                       // the wide launch's shared memory when split
+    int CL2 = 0, WPC2 = 0, L_smem2 = 0;
+    size_t smem2 = 0;
 };
 // Decision bits of every DP kernel, packed by each thread over blocks of 32
 // rows in sweep order (row r = n - 1 - i, block r / 32, bit r % 32): for chain
@@ -82,8 +92,8 @@ struct DpGeom {
 // taken and leaves D[parent+1] = D[next(parent)], so dropping those rows
 // changes no value and no bit of a kept row (see k_prune).
 // For the traceback, per kept row t (kept index, sweep order): skip[t] = kept
-// index of next(row t), -1 when next(row t) = n; skip2[t] = skip[skip[t]]
-// (-1 propagates); wsuf[t] = sum of the weights of kept rows t..nkept-1.
+// index of next(row t), -1 when next(row t) = n; wsuf[t] = sum of the
+// weights of kept rows t..nkept-1.
 struct DpWork {
     uint32_t *bits = nullptr;      // [batch][P][nblk][C][32]
     int32_t *rowlist = nullptr;    // [batch][n]
@@ -91,7 +101,6 @@ struct DpWork {
     int32_t *cnt = nullptr;        // [batch][n + 1]
     int32_t *nkept = nullptr;      // [batch]
     int32_t *skip = nullptr;       // [batch][n]
-    int32_t *skip2 = nullptr;      // [batch][n]
     int32_t *wsuf = nullptr;       // [batch][n + 1]
     int64_t *rowp = nullptr;       // [batch][n] profit of each kept row, sweep order
     int32_t *rowm = nullptr;       // [batch][n] wave-kernel metadata of each kept row
@@ -141,6 +150,10 @@ struct pp_instance {
     pp::Scratch sg;                     // safeguard candidates' working set
     pp::Scratch rp;                     // epoch update working set
     pp::Scratch top2;                   // top-2 holder tables of the planner
+    // split DP launches: the two launches run on these streams (higher and
+    // lower priority), forked from and joined back to the caller's stream
+    cudaStream_t split_hi = nullptr, split_lo = nullptr;
+    cudaEvent_t split_fork = nullptr, split_join_hi = nullptr, split_join_lo = nullptr;
 };
 
 namespace pp {

@@ -359,6 +359,53 @@ def test_single_update_full_size(pp, oracle_lib, cfg):
     np.testing.assert_array_equal(chosen.cpu().numpy()[0], och)
 
 
+@pytest.mark.parametrize("B", [16, 17])
+def test_split_launch_matches_single_launch(pp, oracle_lib, B):
+    """A paper-scale batch just above what clusters of 8 CTAs hold at one CTA
+    per SM runs as two concurrent launches (the smallest sweeps on narrower
+    clusters); optima, decision bits and chosen sets must equal those of one
+    launch of the same shape, and the oracle's on sampled items."""
+    inst = wl.make(3)
+    prob = oracle_lib.Problem.from_instance(inst)
+    rng = np.random.default_rng(77 + B)
+    pls = [_random_feasible_placement(rng, inst, float(f)) for f in (0.0, 0.15, 0.3)]
+    workers = [b % inst.W for b in range(B)]
+    masks = np.zeros((B, inst.n), np.uint32)
+    for b in range(B):
+        pl = pls[b % len(pls)]
+        for m in range(inst.W):
+            if m != workers[b]:
+                masks[b] |= pl[m].astype(np.uint32) << np.uint32(m)
+    k = int(inst.budget[0])
+    with pp.Instance.from_workload(inst) as ppi:
+        split = pp.pp_dp_split(ppi, B, k)
+        if torch.cuda.get_device_properties(0).multi_processor_count == 152:
+            assert split["wide_items"] == 15 and split["narrow_cluster_ctas"] == 4, split
+        prof = torch.zeros((B, inst.n), dtype=torch.int64, device="cuda")
+        pp.pp_marginals(ppi, _dev(workers, np.int32), _dev(masks.view(np.int32), np.int32), prof)
+        bud = _dev(np.full(B, k), np.int32)
+        outs = []
+        for tune in [(0, 0), (8, 4)]:               # automatic (split), then one launch
+            pp.pp_tune_dp(*tune, False, False)
+            try:
+                best = torch.zeros(B, dtype=torch.int64, device="cuda")
+                bits = torch.zeros(pp.pp_dp_bits_size(ppi, B, k) // 4, dtype=torch.int32, device="cuda")
+                chosen = torch.zeros((B, inst.n), dtype=torch.uint8, device="cuda")
+                pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
+                pp.pp_traceback(ppi, bits, bud, k, chosen)
+                ppi.sync()
+            finally:
+                pp.pp_tune_dp(0, 0, False, False)
+            outs.append((best.cpu().numpy(), bits.cpu().numpy(), chosen.cpu().numpy()))
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
+    np.testing.assert_array_equal(outs[0][1], outs[1][1])
+    np.testing.assert_array_equal(outs[0][2], outs[1][2])
+    for b in (0, B - 1):
+        ob, _, och = oracle_lib.worker_update(prob, workers[b], pls[b % len(pls)])
+        assert int(outs[0][0][b]) == ob
+        np.testing.assert_array_equal(outs[0][2][b], och)
+
+
 def test_plan_paper_scale_properties(pp, oracle_lib):
     """The n=50,000 / 16-worker / 16-start plan the benchmark times: every
     target prefix-complete and within budget, objective equal to the oracle's
