@@ -924,8 +924,8 @@ __global__ void __launch_bounds__(1024)
 k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict__ order,
         const int32_t *__restrict__ next, const int2 *__restrict__ pspan,
         const int32_t *__restrict__ wpre, const int32_t *__restrict__ wmeta,
-        const int32_t *__restrict__ item_active, DpWork w, int prune,
-        unsigned long long *__restrict__ rows_kept)
+        const int32_t *__restrict__ item_active, DpWork w, int prune, int wave, int stack_depth,
+        int32_t *__restrict__ status, unsigned long long *__restrict__ rows_kept)
 {
     constexpr int V = 4;
     __shared__ int sh[32];
@@ -983,9 +983,12 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         const int2 sp = pspan[i];
         if (!(sp.x < 0 || cnt[sp.y] - cnt[sp.x] > 0)) return false;
         // an identity row (p <= 0 and no positive strict descendant, so D[i] =
-        // D[next(i)] and every bit is "skip") without a stack operation leaves
-        // the register state unchanged: drop it too
-        return !((wmeta[i] & kWaveStackOps) == 0 && cnt[next[i]] - cnt[i + 1] == 0 && pval(i) <= 0);
+        // D[next(i)] and every bit is "skip") is dropped too: a skip to it
+        // lands on the first kept row after it, which holds the same values.
+        // The one-CTA kernel reads the host's stack plan and keeps the ones
+        // with a stack operation; the wavefront kernel's plan is rebuilt below
+        const bool ident = cnt[next[i]] - cnt[i + 1] == 0 && pval(i) <= 0;
+        return !(ident && (wave || (wmeta[i] & kWaveStackOps) == 0));
     };
     slice(n, lo, hi);
     int kmine = 0, wmine = 0;
@@ -1055,7 +1058,8 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
                 sk[q] = nx < n ? kx[nx] : -1;
                 wq[v] = wpre[i];
                 rp[q] = pval(i);
-                rm[q] = wmeta[i];
+                rm[q] = wmeta[i];               // the wavefront kernel's is rebuilt below
+                if (wave) cnt[q] = -1;          // cnt (done with) becomes last_top_reader
             }
             wl += wq[v];
         }
@@ -1072,6 +1076,79 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         wcarry += tt;
     }
     if (cr == 0 && t == 0) ws[nk] = 0;
+    if (!wave) return;
+
+    // Skip-row stack plan of the wavefront kernel over the kept rows (the
+    // host's plan is for the whole tree; after pruning many of its pushes
+    // have no reader left).  Kept row q reads row sk[q]: the row just
+    // computed when sk[q] = q - 1, else the stack top (the zero row when the
+    // stack is empty, which is the case whenever sk[q] = -1).  A row read
+    // through the stack is pushed when computed and popped after its last
+    // such reader; the rows pushed in between are popped before it, so
+    // every read is of the top.
+    int32_t *lr_ = cnt;                                   // last_top_reader[target]
+    cluster_sync_all();                                   // sk and the -1s complete
+    for (int q = lo + t; q < hi; q += T) {
+        const int s = sk[q];
+        if (s >= 0 && s != q - 1) atomicMax(lr_ + s, q);
+    }
+    cluster_sync_all();                                   // last readers complete
+    auto delta = [&](int q, bool &pop, bool &push) {
+        const int s = sk[q];
+        pop = s >= 0 && s != q - 1 && lr_[s] == q;
+        push = lr_[q] >= 0;
+        return (int)push - (int)pop;
+    };
+    int dmine = 0;
+    for (int q = lo + t; q < hi; q += T) {
+        bool a, b;
+        dmine += delta(q, a, b);
+    }
+    block_exclusive_scan(dmine, &total, sh);
+    int dcarry = cluster_exclusive_scan(total, &total, &slot, bcast);
+    for (int base = lo; base < hi; base += tile) {
+        int dq[V], dl = 0;
+        bool pq[V], uq[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int q = base + t * V + v;
+            dq[v] = 0;
+            pq[v] = uq[v] = false;
+            if (q < hi) dq[v] = delta(q, pq[v], uq[v]);
+            dl += dq[v];
+        }
+        int tt;
+        int ex = block_exclusive_scan(dl, &tt, sh) + dcarry;   // stack depth before row q
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int q = base + t * V + v;
+            if (q < hi) {
+                const int s = sk[q];
+                const int d = ex - (int)pq[v];            // after the pop
+                int flags = 0, lvl = 0;
+                if (uq[v]) {
+                    flags = kWavePush;
+                    lvl = d;
+                } else if (pq[v] && d > 0) {
+                    flags = kWaveReload;                  // the level below becomes the top
+                    lvl = d - 1;
+                } else if (pq[v]) {
+                    flags = kWaveZeroTop;                 // the stack emptied: top = zero row
+                }
+                if ((flags & (kWavePush | kWaveReload)) && lvl >= stack_depth) {
+                    // cannot happen (the plan of an ancestor-closed sub-forest is
+                    // never deeper than the whole tree's): report, stay in bounds
+                    atomicExch(status, (int32_t)PP_EBOUNDS);
+                    flags = 0;
+                    lvl = 0;
+                }
+                const int wq = wpre[rl[q]];
+                rm[q] = wave_pack(wq > 8 ? 8 : wq, s >= 0 && s == q - 1 ? kWaveCur : kWaveTop, flags, lvl);
+                ex += dq[v];
+            }
+        }
+        dcarry += tt;
+    }
 }
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1351,13 +1428,14 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
         pc.numAttrs = 1;
         const int32_t *ord = inst->d_order, *nxt = inst->d_next, *wp = inst->d_wpre, *wm = inst->d_wave;
         const int2 *psp = inst->d_pspan;
-        const int pr = !g_tune_noprune;
+        const int pr = !g_tune_noprune, wv = g.wave, sd = inst->stack_depth;
+        int32_t *stt = inst->d_status;
         if (by_node)
             PP_CUDA(cudaLaunchKernelEx(&pc, k_prune<true>, inst->n, profit, ord, nxt, psp, wp, wm, item_active,
-                                       work, pr, rows_kept));
+                                       work, pr, wv, sd, stt, rows_kept));
         else
             PP_CUDA(cudaLaunchKernelEx(&pc, k_prune<false>, inst->n, profit, ord, nxt, psp, wp, wm, item_active,
-                                       work, pr, rows_kept));
+                                       work, pr, wv, sd, stt, rows_kept));
     }
     PP_CUDA(cudaGetLastError());
     uint32_t *bits = work.bits;

@@ -45,7 +45,7 @@ inline int32_t meta_pack(int skip, int push)
 constexpr int kWaveCur = 0, kWaveTop = 2;
 constexpr int kWaveReload = 1 << 5, kWavePush = 1 << 6, kWaveZeroTop = 1 << 7;
 constexpr int kWaveStackOps = kWaveReload | kWavePush | kWaveZeroTop;
-inline int32_t wave_pack(int w, int kind, int flags, int level)
+__host__ __device__ inline int32_t wave_pack(int w, int kind, int flags, int level)
 {
     return (int32_t)((uint32_t)(w - 1) | ((uint32_t)kind << 3) | (uint32_t)flags | ((uint32_t)level << 16));
 }
