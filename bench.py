@@ -477,7 +477,7 @@ def run_native(args):
             "update_note": "one batched worker update (marginals + tree DP + traceback/accept) of all starts",
             "probes": probes,
             "next_steps": extras,
-            "dp_geometry": pp.pp_dp_geometry(ppi, S, k),
+            "dp_geometry": {**pp.pp_dp_geometry(ppi, S, k), "split": pp.pp_dp_split(ppi, S, k)},
         }
         print(json.dumps(line), flush=True)
     ppi.close()
@@ -509,7 +509,8 @@ def run_profile_dp(args):
         pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
         pp.pp_traceback(ppi, bits, bud, k, chosen)
     ppi.sync()
-    print(json.dumps({"profile_dp": B, "geometry": pp.pp_dp_geometry(ppi, B, k), "best": best.tolist()}))
+    print(json.dumps({"profile_dp": B, "geometry": pp.pp_dp_geometry(ppi, B, k), "split": pp.pp_dp_split(ppi, B, k),
+                      "best": best.tolist()}))
     return 0
 
 
