@@ -161,7 +161,7 @@ __device__ __forceinline__ bool spin_until(Ready ready, int32_t *status)
 
 __host__ __device__ inline size_t wave_fixed_bytes(int WPC, int WMAX)
 {
-    size_t b = (size_t)WPC * wavecfg::kRing * WMAX * sizeof(uint64_t) + (size_t)WPC * 32 * 16 +
+    size_t b = (size_t)WPC * wavecfg::kRing * WMAX * sizeof(uint64_t) + (size_t)WPC * 2 * 32 * 12 +
                (size_t)WPC * sizeof(uint32_t);
     return (b + 15) & ~(size_t)15;
 }
@@ -282,8 +282,9 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
     const int k = kreq < kpad ? kreq : kpad;   // kpad covers min(max_budget, total weight)
 
     uint64_t *ring = reinterpret_cast<uint64_t *>(smem);                           // [WPC][kRing][WMAX]
-    int4 *mstage = reinterpret_cast<int4 *>(ring + (size_t)WPC * kRing * WMAX);    // [WPC][32] (p, m)
-    uint32_t *ack = reinterpret_cast<uint32_t *>(mstage + (size_t)WPC * 32);       // [WPC]
+    int64_t *pstage = reinterpret_cast<int64_t *>(ring + (size_t)WPC * kRing * WMAX);  // [WPC][2][32] profits
+    int32_t *mstage = reinterpret_cast<int32_t *>(pstage + (size_t)WPC * 64);         // [WPC][2][32] metadata
+    uint32_t *ack = reinterpret_cast<uint32_t *>(mstage + (size_t)WPC * 64);          // [WPC]
     int64_t *stk = reinterpret_cast<int64_t *>(smem + wave_fixed_bytes(WPC, WMAX)); // [WPC][L_smem][C][32]
     for (int x = threadIdx.x; x < WPC * kRing * WMAX; x += NT) ring[x] = kLapBit;  // lap of row -1
     if (threadIdx.x < WPC) ack[threadIdx.x] = 0;
@@ -300,7 +301,8 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
         pv_ack = prev_remote ? map_to_rank(la, cr - 1) : la;
     }
     const uint64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
-    int4 *my_meta = mstage + (size_t)wl * 32;
+    int64_t *const my_ps = pstage + (size_t)wl * 64;
+    int32_t *const my_ms = mstage + (size_t)wl * 64;
     const uint32_t my_ack = smem_addr(ack + wl);
     uint32_t ack_seen = 0;
     bool aborted = false;
@@ -326,35 +328,39 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
         cur[c] = 0;          // row n is the zero boundary, and the top of the empty stack
         top[c] = 0;
     }
-    // row metadata, 32 rows per block: lane l loads row blk*32 + l one block
-    // ahead; the warp stages the profits (and stack levels) in shared memory
-    // and turns the flags into warp-uniform masks, bit = row of the block.
-    // Rows past the last one are no-ops (p = -inf, skip = the row just
-    // computed), so every warp sweeps nblk_item * 32 rows.
-    auto load_meta = [&](int r, int64_t &pv, int32_t &mv) {
+    // row metadata, 32 rows per block: lane l copies row blk*32 + l one block
+    // ahead into a double buffer in shared memory with cp.async (a register
+    // load in flight across the rows held a scoreboard that the rows' own
+    // waits then also waited on); the warp turns the flags into warp-uniform
+    // masks, bit = row of the block.  Rows past the last one are no-ops
+    // (p = -inf, skip = the row just computed), so every warp sweeps
+    // nblk_item * 32 rows.
+    auto prefetch = [&](int b) {
+        const int r = b * 32 + lane, o = (b & 1) * 32 + lane;
         if (r < nrows) {
-            pv = Rp[r];         // one independent load each: nothing waits
-            mv = Rm[r];         // for them before the next block
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_addr(my_ps + o)),
+                         "l"(__cvta_generic_to_global(Rp + r)) : "memory");
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(my_ms + o)),
+                         "l"(__cvta_generic_to_global(Rm + r)) : "memory");
         } else {
-            pv = kNeg;
-            mv = 0;
+            my_ps[o] = kNeg;
+            my_ms[o] = 0;
         }
+        asm volatile("cp.async.commit_group;" ::: "memory");
     };
-    int64_t pnext;
-    int32_t mnext;
-    load_meta(lane, pnext, mnext);
+    prefetch(0);
     // boundary carried between sub-blocks: D[i+1][base - WMAX + 1 + q] of the
     // previous warp for the first row of the next sub-block (row n: zeros)
     int64_t carry[WMAX];
 #pragma unroll
     for (int q = 0; q < WMAX; ++q) carry[q] = has_prev ? 0 : (q == WMAX - 1 ? 0 : kNeg);
-    int64_t *const my_p = reinterpret_cast<int64_t *>(my_meta);     // [32] profits of the block
-    int32_t *const my_lv = reinterpret_cast<int32_t *>(my_p + 32);  // [32] stack levels
 
     for (int blk = 0; blk < nblk_item && !aborted; ++blk) {
+        asm volatile("cp.async.wait_all;" ::: "memory");
         __syncwarp();
-        my_p[lane] = pnext;
-        my_lv[lane] = (int32_t)((uint32_t)mnext >> 16);
+        const int64_t *const my_p = my_ps + (blk & 1) * 32;      // [32] profits of the block
+        const int32_t *const my_m = my_ms + (blk & 1) * 32;      // [32] metadata of the block
+        const int32_t mnext = my_m[lane];
         const uint32_t cur_rows = __ballot_sync(kFull, (mnext & (3 << 3)) == (kWaveCur << 3));
         const uint32_t push_rows = __ballot_sync(kFull, (mnext & kWavePush) != 0);
         const uint32_t reload_rows = __ballot_sync(kFull, (mnext & kWaveReload) != 0);
@@ -364,8 +370,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             w1_rows = __ballot_sync(kFull, (mnext & 1) != 0);
             w2_rows = __ballot_sync(kFull, (mnext & 2) != 0);
         }
-        __syncwarp();
-        load_meta((blk + 1) * 32 + lane, pnext, mnext);
+        if (blk + 1 < nblk_item) prefetch(blk + 1);     // the other buffer: block blk - 1 is done
         uint32_t wbits[C];
 #pragma unroll
         for (int c = 0; c < C; ++c) wbits[c] = 0;
@@ -467,7 +472,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                 // the top), reload the new top after a pop, or reset it to the zero row
                 if (STACK && ((stk8 >> u) & 1u)) {
                     if ((pb >> u) & 1u) {
-                        const int lvl = my_lv[s8 + u];
+                        const int lvl = (int)((uint32_t)my_m[s8 + u] >> 16);
 #pragma unroll
                         for (int c = 0; c < C; ++c) top[c] = cur[c];
                         if (lvl < L_smem) {
@@ -478,7 +483,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                             for (int c = 0; c < C; ++c) my_gst[(size_t)(lvl - L_smem) * CL * C * NT + (size_t)c * NT] = cur[c];
                         }
                     } else if ((rb >> u) & 1u) {
-                        const int lvl = my_lv[s8 + u];
+                        const int lvl = (int)((uint32_t)my_m[s8 + u] >> 16);
                         if (lvl < L_smem) {
 #pragma unroll
                             for (int c = 0; c < C; ++c) top[c] = my_stk[((size_t)lvl * C + c) * 32];
@@ -526,6 +531,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
         for (int c = 0; c < C; ++c) Bw[((size_t)blk * C + c) * 32] = wbits[c];
     }
 
+    asm volatile("cp.async.wait_all;" ::: "memory");   // nothing in flight into this CTA's shared memory
     if (!aborted) {
         if (k == 0) {
             if (g == 0 && lane == 0) best[item] = 0;
