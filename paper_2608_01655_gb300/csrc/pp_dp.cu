@@ -15,11 +15,11 @@
 //   Every warp sweeps its own columns row after row; warp g needs, for row i,
 //   the last w_i values of row i+1 of warp g-1, which that warp publishes
 //   into a ring in warp g's shared memory (DSMEM when g-1 is in the previous
-//   CTA of the cluster).  Ring counters are published with release stores
-//   every kPub rows and read with acquire loads; the consumer acknowledges
-//   slots so the producer never overwrites an unread one.  So warps form a
-//   wavefront, warp g lagging warp g-1 by a few rows.  Every wait is bounded
-//   in time and reports PP_ETIMEOUT through the status word.
+//   CTA of the cluster).  Each slot carries a lap bit, so a slot validates
+//   itself and no fence is needed; the consumer acknowledges finished rows so
+//   the producer never overwrites an unread slot.  So warps form a wavefront,
+//   warp g lagging warp g-1 by a sub-block of rows.  Every wait is bounded in
+//   time and reports PP_ETIMEOUT through the status word.
 // k_tree_dp_flat (any weight): one CTA per DP, row i+1 staged in shared memory
 //   and one __syncthreads per row.
 //
@@ -109,15 +109,15 @@ __device__ __forceinline__ uint32_t ld_relaxed_cluster_u32(uint32_t addr)
     asm volatile("ld.relaxed.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
     return v;
 }
-__device__ __forceinline__ void st_relaxed_cluster_u64_if(bool pred, uint32_t addr, uint64_t v)
-{
-    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %0, 0;\n\t"
-                 "@p st.relaxed.cluster.shared::cluster.u64 [%1], %2;\n\t}"
-                 ::"r"((uint32_t)pred), "r"(addr), "l"(v));
-}
 __device__ __forceinline__ void ld_volatile_v2_u64(const uint64_t *p, uint64_t &a, uint64_t &b)
 {
     asm volatile("ld.volatile.shared.v2.u64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(smem_addr(p)) : "memory");
+}
+__device__ __forceinline__ volatile uint64_t *map_generic_u64(const void *p, uint32_t rank)
+{
+    uint64_t r;
+    asm volatile("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(p), "r"(rank));
+    return reinterpret_cast<volatile uint64_t *>(r);
 }
 __device__ __forceinline__ uint64_t global_ns()
 {
@@ -292,15 +292,17 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
 
     const bool has_prev = g > 0, has_next = g < P - 1;
     const bool prev_remote = has_prev && wl == 0;
-    // the next warp's ring through the cluster window (local or remote alike)
-    const uint32_t nx_ring = has_next ? map_to_rank(smem_addr(ring + (size_t)((wl + 1) % WPC) * kRing * WMAX),
-                                                    (uint32_t)(wl == WPC - 1 ? cr + 1 : cr)) : 0u;
     uint32_t pv_ack = 0;
     if (has_prev) {
         const uint32_t la = smem_addr(ack + (prev_remote ? WPC - 1 : wl - 1));
         pv_ack = prev_remote ? map_to_rank(la, cr - 1) : la;
     }
     const uint64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
+    // the next warp's ring through the cluster window (local or remote alike),
+    // as a generic address: a plain volatile store lets the compiler schedule
+    // the rows around the hand-off (an inline-PTX store cost ~5% per row)
+    volatile uint64_t *const nx_gen = has_next ? map_generic_u64(ring + (size_t)((wl + 1) % WPC) * kRing * WMAX,
+                                                                 (uint32_t)(wl == WPC - 1 ? cr + 1 : cr)) : nullptr;
     int64_t *const my_ps = pstage + (size_t)wl * 64;
     int32_t *const my_ms = mstage + (size_t)wl * 64;
     const uint32_t my_ack = smem_addr(ack + wl);
@@ -378,13 +380,6 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             const int r0 = blk * 32 + sb * kSub;
             // producer: slots r0..r0+kSub-1 last held rows r0-kRing.., which the
             // consumer has finished reading once it reports row r0+kSub+1-kRing
-            if (has_next && r0 + kSub + 1 > kRing && ack_seen < (uint32_t)(r0 + kSub + 1 - kRing)) {
-                const uint32_t need = (uint32_t)(r0 + kSub + 1 - kRing);
-                if (!spin_until([&] { ack_seen = ld_relaxed_cluster_u32(my_ack); return ack_seen >= need; }, status)) {
-                    aborted = true;
-                    break;
-                }
-            }
             // consumer: rows r0..r0+kSub-1 of the previous warp, all with the
             // lap bit of this pass over the ring
             const uint64_t lap = (uint64_t)((r0 / kRing) & 1) << 63;
@@ -392,8 +387,16 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             uint64_t sv[WMAX == 1 ? kSub : 1];
 #pragma unroll
             for (int u = 0; u < (WMAX == 1 ? kSub : 1); ++u) sv[u] = 0;
-            if (has_prev) {
+            const bool need_ack = has_next && r0 + kSub + 1 > kRing && ack_seen < (uint32_t)(r0 + kSub + 1 - kRing);
+            if (has_prev || need_ack) {
+                const uint32_t need = (uint32_t)(r0 + kSub + 1 - kRing);
                 auto ready = [&] {
+                    bool ok = true;
+                    if (need_ack) {
+                        ack_seen = ld_relaxed_cluster_u32(my_ack);
+                        ok = ack_seen >= need;
+                    }
+                    if (!has_prev) return ok;
                     uint64_t bad = 0;
                     if (WMAX == 1) {
 #pragma unroll
@@ -412,7 +415,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                             bad |= (x ^ lap) | (y ^ lap);
                         }
                     }
-                    return (bad & kLapBit) == 0;
+                    return ok && (bad & kLapBit) == 0;
                 };
                 if (!spin_until(ready, status)) {
                     aborted = true;
@@ -423,7 +426,6 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             const uint32_t cb = cur_rows >> s8, pb = push_rows >> s8, rb = reload_rows >> s8;
             const uint32_t stk8 = ((push_rows | reload_rows | zero_rows) >> s8) & ((1u << kSub) - 1);
             const uint32_t wb1 = w1_rows >> s8, wb2 = w2_rows >> s8;
-            const uint32_t sa0 = nx_ring + (uint32_t)((r0 & (kRing - 1)) * WMAX * 8);
             uint32_t wb8[C];
 #pragma unroll
             for (int c = 0; c < C; ++c) wb8[c] = 0;
@@ -466,8 +468,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                 // hand this row's last WMAX columns to the next warp (lane 31 only)
 #pragma unroll
                 for (int q = 0; q < WMAX; ++q)
-                    st_relaxed_cluster_u64_if(publish, sa0 + (uint32_t)((u * WMAX + q) * 8),
-                                              (uint64_t)cur[C - WMAX + q] | lap);
+                    if (publish) nx_gen[(r0 & (kRing - 1)) * WMAX + u * WMAX + q] = (uint64_t)cur[C - WMAX + q] | lap;
                 // skip-row stack (warp-uniform masks): push (the new row becomes
                 // the top), reload the new top after a pop, or reset it to the zero row
                 if (STACK && ((stk8 >> u) & 1u)) {
