@@ -71,53 +71,16 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank)
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
-__device__ __forceinline__ void st_cluster_s64(uint32_t addr, int64_t v)
-{
-    asm volatile("st.shared::cluster.s64 [%0], %1;" ::"r"(addr), "l"(v) : "memory");
-}
-__device__ __forceinline__ void st_release_cluster_u32(uint32_t addr, uint32_t v)
-{
-    asm volatile("st.release.cluster.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ void st_release_cta_u32(uint32_t addr, uint32_t v)
-{
-    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t ld_acquire_cluster_u32(uint32_t addr)
-{
-    uint32_t v;
-    asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-    return v;
-}
-__device__ __forceinline__ void st_relaxed_cluster_u64(uint32_t addr, uint64_t v)
-{
-    asm volatile("st.relaxed.cluster.shared::cluster.u64 [%0], %1;" ::"r"(addr), "l"(v) : "memory");
-}
-__device__ __forceinline__ void st_relaxed_cluster_u32(uint32_t addr, uint32_t v)
-{
-    asm volatile("st.relaxed.cluster.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint64_t ld_relaxed_cluster_u64(uint32_t addr)
-{
-    uint64_t v;
-    asm volatile("ld.relaxed.cluster.shared::cta.u64 %0, [%1];" : "=l"(v) : "r"(addr) : "memory");
-    return v;
-}
-__device__ __forceinline__ uint32_t ld_relaxed_cluster_u32(uint32_t addr)
-{
-    uint32_t v;
-    asm volatile("ld.relaxed.cluster.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-    return v;
-}
 __device__ __forceinline__ void ld_volatile_v2_u64(const uint64_t *p, uint64_t &a, uint64_t &b)
 {
     asm volatile("ld.volatile.shared.v2.u64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(smem_addr(p)) : "memory");
 }
-__device__ __forceinline__ volatile uint64_t *map_generic_u64(const void *p, uint32_t rank)
+// generic address of `p` (this CTA's shared memory) in CTA `rank` of the cluster
+__device__ __forceinline__ void *map_generic(const void *p, uint32_t rank)
 {
     uint64_t r;
     asm volatile("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(p), "r"(rank));
-    return reinterpret_cast<volatile uint64_t *>(r);
+    return reinterpret_cast<void *>(r);
 }
 __device__ __forceinline__ uint64_t global_ns()
 {
@@ -292,20 +255,19 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
 
     const bool has_prev = g > 0, has_next = g < P - 1;
     const bool prev_remote = has_prev && wl == 0;
-    uint32_t pv_ack = 0;
-    if (has_prev) {
-        const uint32_t la = smem_addr(ack + (prev_remote ? WPC - 1 : wl - 1));
-        pv_ack = prev_remote ? map_to_rank(la, cr - 1) : la;
-    }
+    // the previous warp's acknowledgement word, as a generic cluster address
+    volatile uint32_t *pv_ack = nullptr;
+    if (has_prev)
+        pv_ack = reinterpret_cast<volatile uint32_t *>(
+            map_generic(ack + (prev_remote ? WPC - 1 : wl - 1), (uint32_t)(prev_remote ? cr - 1 : cr)));
     const uint64_t *my_ring = ring + (size_t)wl * kRing * WMAX;
     // the next warp's ring through the cluster window (local or remote alike),
     // as a generic address: a plain volatile store lets the compiler schedule
     // the rows around the hand-off (an inline-PTX store cost ~5% per row)
-    volatile uint64_t *const nx_gen = has_next ? map_generic_u64(ring + (size_t)((wl + 1) % WPC) * kRing * WMAX,
+    volatile uint64_t *const nx_gen = has_next ? (volatile uint64_t *)map_generic(ring + (size_t)((wl + 1) % WPC) * kRing * WMAX,
                                                                  (uint32_t)(wl == WPC - 1 ? cr + 1 : cr)) : nullptr;
     int64_t *const my_ps = pstage + (size_t)wl * 64;
     int32_t *const my_ms = mstage + (size_t)wl * 64;
-    const uint32_t my_ack = smem_addr(ack + wl);
     uint32_t ack_seen = 0;
     bool aborted = false;
     const bool publish = has_next && lane == 31 && g != g_drop_publish_warp;   // this lane stores
@@ -393,7 +355,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                 auto ready = [&] {
                     bool ok = true;
                     if (need_ack) {
-                        ack_seen = ld_relaxed_cluster_u32(my_ack);
+                        ack_seen = *(volatile uint32_t *)(ack + wl);
                         ok = ack_seen >= need;
                     }
                     if (!has_prev) return ok;
@@ -522,10 +484,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                     for (int q = 0; q < WMAX; ++q) carry[q] = (int64_t)(sl[(kSub - 1) * WMAX + q] & ~kLapBit);
                 }
                 // report the finished rows to the previous warp (values already used)
-                if (lane == 0) {
-                    if (prev_remote) st_relaxed_cluster_u32(pv_ack, (uint32_t)(r0 + kSub));
-                    else *(volatile uint32_t *)(ack + wl - 1) = (uint32_t)(r0 + kSub);
-                }
+                if (lane == 0) *pv_ack = (uint32_t)(r0 + kSub);
             }
         }
 #pragma unroll
