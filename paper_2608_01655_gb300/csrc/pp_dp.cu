@@ -190,7 +190,7 @@ __device__ __forceinline__ void shift_row(const int64_t (&cur)[C], const int64_t
 constexpr int kSub = wavecfg::kPub;
 constexpr uint64_t kLapBit = 1ull << 63;
 
-template <int C, int WMAX>
+template <int C, int WMAX, bool SPILL>
 __global__ void __launch_bounds__(512, 1)
 k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                const int32_t *__restrict__ rowm, const int32_t *__restrict__ nkept,
@@ -438,7 +438,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                         const int lvl = (int)((uint32_t)my_m[s8 + u] >> 16);
 #pragma unroll
                         for (int c = 0; c < C; ++c) top[c] = cur[c];
-                        if (lvl < L_smem) {
+                        if (!SPILL || lvl < L_smem) {
 #pragma unroll
                             for (int c = 0; c < C; ++c) my_stk[((size_t)lvl * C + c) * 32] = cur[c];
                         } else {
@@ -447,7 +447,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                         }
                     } else if ((rb >> u) & 1u) {
                         const int lvl = (int)((uint32_t)my_m[s8 + u] >> 16);
-                        if (lvl < L_smem) {
+                        if (!SPILL || lvl < L_smem) {
 #pragma unroll
                             for (int c = 0; c < C; ++c) top[c] = my_stk[((size_t)lvl * C + c) * 32];
                         } else {
@@ -1155,11 +1155,16 @@ DpWork dp_work_split(void *base, int batch, int n, int words)
 // geometry and launch
 // ===========================================================================
 template <int C, int WMAX>
-static const void *wave_kernel() { return (const void *)k_tree_dp_wave<C, WMAX>; }
-
-static const void *wave_kernel_for(int C, int WMAX)
+static const void *wave_kernel(bool spill)
 {
-#define PP_WAVE_CASE(CC, WW) if (C == CC && WMAX == WW) return wave_kernel<CC, WW>();
+    return spill ? (const void *)k_tree_dp_wave<C, WMAX, true> : (const void *)k_tree_dp_wave<C, WMAX, false>;
+}
+
+// spill: some skip-row stack levels live in global memory (the kernel without
+// that branch is ~5% faster per row)
+static const void *wave_kernel_for(int C, int WMAX, bool spill)
+{
+#define PP_WAVE_CASE(CC, WW) if (C == CC && WMAX == WW) return wave_kernel<CC, WW>(spill);
     PP_WAVE_CASE(1, 1) PP_WAVE_CASE(2, 1) PP_WAVE_CASE(4, 1) PP_WAVE_CASE(8, 1)
     PP_WAVE_CASE(2, 2) PP_WAVE_CASE(4, 2) PP_WAVE_CASE(8, 2)
     PP_WAVE_CASE(4, 4) PP_WAVE_CASE(8, 4)
@@ -1210,8 +1215,8 @@ static void split_geometry(const pp_instance *inst, int batch, const void *fn, c
     if (fixed2 > (size_t)smem_max) return;
     const int L2 = (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed2) / level2);
     const size_t smem2 = std::max(fixed2 + (size_t)L2 * level2, excl);
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)std::max(excl, smem2)) !=
-        cudaSuccess) {
+    const void *fn2 = wave_kernel_for(g->C, g->WMAX, L2 < inst->stack_depth);
+    if (!fn2 || cudaFuncSetAttribute(fn2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2) != cudaSuccess) {
         cudaGetLastError();
         return;
     }
@@ -1227,7 +1232,7 @@ static void split_geometry(const pp_instance *inst, int batch, const void *fn, c
     cfg2.attrs = attr;
     cfg2.numAttrs = 1;
     int m2 = 0;
-    if (cudaOccupancyMaxActiveClusters(&m2, fn, &cfg2) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&m2, fn2, &cfg2) != cudaSuccess) {
         cudaGetLastError();
         return;
     }
@@ -1263,12 +1268,12 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
         if (g_tune_c > 0) C = std::max(std::min(g_tune_c, 8), WMAX);
         const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
         if (WPC > 16) continue;
-        const void *fn = wave_kernel_for(C, WMAX);
-        if (!fn) continue;
         const size_t fixed = wave_fixed_bytes(WPC, WMAX);
         const size_t level = (size_t)C * WPC * 32 * sizeof(int64_t);
         if (fixed > (size_t)smem_max) continue;
         const int L_smem = (int)std::min<size_t>((size_t)inst->stack_depth, ((size_t)smem_max - fixed) / level);
+        const void *fn = wave_kernel_for(C, WMAX, L_smem < inst->stack_depth);
+        if (!fn) continue;
         const size_t smem = fixed + (size_t)L_smem * level;
         if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) {
             cudaGetLastError();
@@ -1407,10 +1412,6 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
     uint32_t *bits = work.bits;
     const int32_t *nkept = work.nkept;
     if (g.wave) {
-        const void *fn = wave_kernel_for(g.C, g.WMAX);
-        if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
-        PP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)(g.split ? std::max(g.smem_x, g.smem2) : g.smem)));
         int32_t n = inst->n;
         int32_t nblk = (n + 31) / 32;
         const int64_t *rowp = work.rowp;
@@ -1419,6 +1420,9 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
         int32_t nb = batch;
         auto launch = [&](int CL, int WPC, size_t smem, int32_t L_smem, int items, int32_t slot_base,
                           cudaStream_t s) -> pp_status {
+            const void *fn = wave_kernel_for(g.C, g.WMAX, L_smem < inst->stack_depth);
+            if (!fn) return fail(PP_EINVAL, "unsupported DP geometry");
+            PP_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
             cudaLaunchConfig_t cfg = {};
             cfg.gridDim = dim3(CL * items);
             cfg.blockDim = dim3(WPC * 32);
