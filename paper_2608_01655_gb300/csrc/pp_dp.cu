@@ -808,21 +808,21 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
 }
 
 // ===========================================================================
-// Pruned sweep (one CTA per item).  A strict descendant set with no positive
-// profit is never worth taking: for a parent x whose strict descendants all
-// have p <= 0, D[x+1][.] = D[next(x)][.] (selecting nothing below x is
-// optimal), every decision bit below x is "skip", and the stack pushes and
-// pops of those rows balance.  So the rows strictly below x can be removed
-// from the sweep: row x then sees D[next(x)] as its row i+1, which is the same
-// values, and no kept row's value or bit changes.  With `cnt` the prefix
-// counts of positive profits in preorder, x has a positive strict descendant
-// iff cnt[next(x)] - cnt[x + 1] > 0, and row i is kept iff it is a root or its
-// parent has one.  A kept row i that is itself an identity (p_i <= 0 and no
-// positive strict descendant: D[i] = D[next(i)] = the row just computed, all
-// bits "skip") and has no skip-row stack operation is dropped as well.  Kept
-// rows are listed in sweep order (decreasing i); every position records the
-// first kept row at or after it in preorder, so a skip to a dropped row lands
-// where the all-"skip" walk through it would.
+// Pruned sweep (one cluster of CTAs per item).  A strict descendant set with
+// no positive profit is never worth taking: for a parent x whose strict
+// descendants all have p <= 0, D[x+1][.] = D[next(x)][.] (selecting nothing
+// below x is optimal) and every decision bit below x is "skip".  So the rows
+// strictly below x can be removed from the sweep: row x then sees D[next(x)]
+// as its row i+1, which is the same values, and no kept row's value or bit
+// changes.  With `cnt` the prefix counts of positive profits in preorder, x
+// has a positive strict descendant iff cnt[next(x)] - cnt[x + 1] > 0, and row
+// i is kept iff it is a root or its parent has one.  A kept row i that is
+// itself an identity (p_i <= 0 and no positive strict descendant: D[i] =
+// D[next(i)], all bits "skip") is dropped as well (for the one-CTA kernel,
+// which follows the host's stack plan, only if it has no stack operation).
+// Kept rows are listed in sweep order (decreasing i); every position records
+// the first kept row at or after it in preorder, so a skip to a dropped row
+// lands where the all-"skip" walk through it would.
 // ===========================================================================
 __device__ __forceinline__ int block_exclusive_scan(int v, int *total, int *sh)
 {
