@@ -87,6 +87,38 @@ def test_tree_dp_and_traceback_small(pp, oracle_lib):
         ppi.close()
 
 
+def test_tree_dp_without_pruning(pp, oracle_lib):
+    """The sweep over every row (pruning off: the prune kernel then only
+    plans the skip-row stack for the whole tree) gives the oracle's optimum
+    and set, as the pruned sweep does, on trees with deep stacks and
+    zero-profit subtrees."""
+    rng = np.random.default_rng(321)
+    trees = _trees(rng)[:8]
+    trees.append(np.array([-1] + [(v - 1) // 3 for v in range(1, 400)], np.int32))      # ternary
+    for parent in trees:
+        n = len(parent)
+        weight = rng.integers(1, 3, size=n).astype(np.int32)
+        ppi = _tree_instance(pp, parent, weight)
+        profits = rng.integers(-2, 9, size=(3, n)).astype(np.int64)
+        profits[1][rng.random(n) < 0.6] = 0
+        tw = int(weight.sum())
+        budgets = np.array([tw // 2 + 1, tw, max(tw // 5, 1)], np.int32)
+        maxb = int(budgets.max())
+        outs = []
+        for no_prune in (True, False):
+            pp.pp_tune_dp(0, 0, False, no_prune)
+            try:
+                outs.append(_dp_batch(pp, ppi, profits, budgets, maxb))
+            finally:
+                pp.pp_tune_dp(0, 0, False, False)
+        for b in range(3):
+            ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+            for best, chosen in outs:
+                assert best[b] == ob, (n, b)
+                np.testing.assert_array_equal(chosen[b], oc)
+        ppi.close()
+
+
 @pytest.mark.parametrize("n,wmax,kmax", [(700, 4, 1500), (3000, 4, 5000), (2500, 1, 2047),
                                          (5000, 3, 9000), (1200, 1, 1061)])
 def test_tree_dp_multi_column_tiles(pp, oracle_lib, n, wmax, kmax):

@@ -66,7 +66,7 @@ def _run(pp, ppi, fn, profits, budgets, k):
 
 
 @pytest.mark.parametrize("w_max,tune", [(6, (0, 0)), (1, (1, 8))])
-def test_noalloc_matches_tree_dp_twice(pp, w_max, tune):
+def test_noalloc_matches_tree_dp_twice(pp, oracle_lib, w_max, tune):
     rng = np.random.default_rng(900 + w_max)
     parent, weight = _deep_stack_tree(rng, 60, 3000, w_max)
     k = 4096
@@ -82,6 +82,11 @@ def test_noalloc_matches_tree_dp_twice(pp, w_max, tune):
             profits[:, rng.random(len(parent)) < 0.3] = 0
             ref = _run(pp, ppi, pp.pp_tree_dp, profits, budgets, k)
             got = _run(pp, ppi, pp.pp_tree_dp_noalloc, profits, budgets, k)
+            if call == 0:                   # the spilling launch against the oracle itself
+                for b in range(2):
+                    ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+                    assert int(ref[0][b]) == ob
+                    np.testing.assert_array_equal(ref[2][b], oc)
             np.testing.assert_array_equal(got[0], ref[0])
             np.testing.assert_array_equal(got[1], ref[1])
             np.testing.assert_array_equal(got[2], ref[2])
