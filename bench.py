@@ -275,9 +275,10 @@ def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, s
 
 def _extras(pp, torch, wl, inst, res):
     """Timings of the steps next to the plan (outside the timed region):
-    the requester-side safeguard candidates on the RAG workload, and one epoch
+    the requester-side safeguard candidates on the RAG workload, one epoch
     update of the paper-scale plan after a popularity shift (log-normal
-    sigma = 0.5 on every demand entry, as in RQ5)."""
+    sigma = 0.5 on every demand entry, as in RQ5), and the plan at the
+    paper's runtime-study budget (k = 128)."""
     out = {}
     rag = wl.make(1)
     with pp.Instance.from_workload(rag) as ppr:
@@ -305,6 +306,19 @@ def _extras(pp, torch, wl, inst, res):
                            "incumbent_objective": rr.incumbent_objective, "new_objective": rr.new_objective,
                            "materialization_cost_us": rr.materialization_cost,
                            "break_even_requests": rr.break_even_requests, "adopted_at_one_epoch": rr.adopted}
+    # the paper's runtime study shape (Fig. 7: n = 50,000, M = 16, k = 128 per
+    # worker, 12.29 s for its CPU solver) on the same synthetic workload
+    small = wl.Instance(**{**inst.__dict__, "budget": np.full(inst.W, 128, np.int32)})
+    with pp.Instance.from_workload(small) as ppk:
+        pp.pp_plan_run(ppk, small.starts, None, small.rounds)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        rk = pp.pp_plan_run(ppk, small.starts, None, small.rounds)
+        t_k = time.perf_counter() - t0
+    out["paper_runtime_shape"] = {"workload": "paper-n50000-W16-k128", "starts": small.starts,
+                                  "rounds": small.rounds, "ms": 1000 * t_k, "objective": rk.objective,
+                                  "context": "the paper's CPU solver: 12.29 s on one EPYC 9V74 (Fig. 7); "
+                                             "starts, objective variant and safeguards not stated there"}
     return out
 
 

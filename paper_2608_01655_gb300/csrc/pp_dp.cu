@@ -1251,22 +1251,32 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     const int smem_max = max_smem_optin(inst);
     int per_item = inst->sm_count / std::max(batch, 1);
     per_item = std::max(1, std::min(8, per_item));
-    const int64_t max_cl = std::max<int64_t>(1, (k + 32 * WMAX - 1) / (32 * WMAX));
-    int cl_hi = (int)std::min<int64_t>(per_item, max_cl);
+    int cl_hi = per_item;
     if (g_tune_cl > 0) cl_hi = std::min(g_tune_cl, 8);
-    // Shape chosen by timing whole plans (paper-scale and source-dependent
-    // workloads): the widest cluster the SMs per item allow, then columns per
-    // thread grown until a CTA has at most 4 warps, but to at most 4 columns
-    // (8 columns per thread cost more than the extra warps).  A batch just
-    // above the number of such clusters that fit at one CTA per SM is split
-    // (split_geometry).
+    // Shape chosen by timing whole plans of the paper-scale workload at budgets
+    // 128 to 4,096: 2 columns per thread (1 and 4 were slower) unless that
+    // needs more than 32 warps per DP, then 4; a budget of at most 128 columns
+    // on a single warp (no hand-off at all); the warps spread over the widest
+    // cluster the SMs per item allow, so that a CTA holds at most 4 warps
+    // while the DP has at most 32 (with 1 or 2 warps per CTA most hand-offs
+    // cross CTAs, which cost more).  A batch just above the number of such
+    // clusters that fit at one CTA per SM is split (split_geometry).
+    int C = WMAX;
+    bool one_warp = false;
+    if (g_tune_c > 0) {
+        C = std::max(std::min(g_tune_c, 8), WMAX);
+    } else if (k <= 128) {
+        while (32 * C < k) C *= 2;
+        one_warp = g_tune_cl <= 0;
+    } else {
+        C = std::max(WMAX, 2);
+        if ((k + 32 * C - 1) / (32 * C) > 32 && C < 4) C = 4;
+        if ((k + 32 * C - 1) / (32 * C) > 128) C = 8;
+    }
+    const int64_t P = (k + 32 * C - 1) / (32 * C);     // warps per DP
+    if (g_tune_cl <= 0) cl_hi = (int)std::min<int64_t>(one_warp ? 1 : cl_hi, P);
     for (int CL = cl_hi; CL >= 1; --CL) {
-        const int64_t cols = (k + CL - 1) / CL;
-        int C = WMAX;
-        while ((cols + 32 * C - 1) / (32 * C) > 4 && C < 4) C *= 2;
-        if ((cols + 32 * C - 1) / (32 * C) > 16) C = 8;
-        if (g_tune_c > 0) C = std::max(std::min(g_tune_c, 8), WMAX);
-        const int WPC = (int)((cols + 32 * C - 1) / (32 * C));
+        const int WPC = (int)((P + CL - 1) / CL);
         if (WPC > 16) continue;
         const size_t fixed = wave_fixed_bytes(WPC, WMAX);
         const size_t level = (size_t)C * WPC * 32 * sizeof(int64_t);
