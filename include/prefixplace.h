@@ -204,7 +204,11 @@ size_t pp_dp_bits_size(const pp_instance *inst, int32_t batch, int32_t max_budge
  *                 bytes, out: decision bits for pp_traceback
  * A budget outside [0, max_budget] sets PP_EBOUNDS and that item's best to 0.
  * The call may allocate instance-owned device scratch for the skip-row stack
- * on first use (or when a larger batch needs more).
+ * on first use (or when a larger batch needs more).  A batch that pp_dp_split
+ * splits runs as two launches on two streams of the instance (created on the
+ * first such call, with three events), forked from and joined back to
+ * `stream`, so the work stays ordered on `stream`; calls on one instance use
+ * its scratch and must not overlap on the GPU.
  */
 pp_status pp_tree_dp(pp_instance *inst, int32_t batch, const int64_t *profit,
                      const int32_t *budget, int32_t max_budget, int64_t *best,
