@@ -680,6 +680,7 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 constexpr int kPruneCluster = 8;         // CTAs per item of the pruned-sweep kernel
 constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (a multiple of 32)
 
+template <int SKIPS>
 __global__ void __launch_bounds__(256)
 k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
@@ -777,13 +778,21 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int pos = pick(rlv, lr, lr & 31);
             const int skr = pick(skv, lr, lr & 31);
             // speculation for the lane that ends the take-run: its skip lands
-            // on row skr at the same column; when that row is in the tile and
+            // on row skr at the same column; while that row is in the tile and
             // is skipped as well, the walk goes on to its skip target in the
-            // same step (skips often come in pairs: ~35% fewer steps)
-            const int lr1 = (skr - r0) & (kTraceTileRows - 1);
-            const uint32_t word1 = (uint32_t)pick(wv, lr1, (j0 - col) & 31);
-            const int sk1 = pick(skv, lr1, lr1 & 31);
-            const int tnext = (skr >= r0 && !((word1 >> (lr1 & 31)) & 1u)) ? sk1 : skr;
+            // same step, up to SKIPS times (skips often come in pairs: with one,
+            // ~35% fewer steps at the paper-scale workload; trees with wide
+            // fan-out have longer runs and use three)
+            int tnext = skr;
+            bool more = true;
+#pragma unroll
+            for (int d = 0; d < SKIPS; ++d) {
+                const int lr1 = (tnext - r0) & (kTraceTileRows - 1);
+                const uint32_t word1 = (uint32_t)pick(wv, lr1, (j0 - col) & 31);
+                const int sk1 = pick(skv, lr1, lr1 & 31);
+                more = more && tnext >= r0 && !((word1 >> (lr1 & 31)) & 1u);
+                tnext = more ? sk1 : tnext;
+            }
             if (lane < L) {
                 if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
                 else chosen[(size_t)item * n + order[pos]] = 1;
@@ -1512,8 +1521,12 @@ pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, con
     if (batch <= 0 || inst->n == 0) return PP_OK;
     AcceptArgs a;
     if (acc) a = *acc;
-    k_traceback<<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
-                                       inst->d_order, chosen, a);
+    if (inst->trace_skips >= 3)
+        k_traceback<3><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
+                                              inst->d_order, chosen, a);
+    else
+        k_traceback<1><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
+                                              inst->d_order, chosen, a);
     PP_CUDA(cudaGetLastError());
     return PP_OK;
 }

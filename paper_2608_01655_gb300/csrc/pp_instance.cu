@@ -295,6 +295,20 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
         inst->total_weight += weight[i];
         inst->max_weight = std::max(inst->max_weight, weight[i]);
     }
+    {
+        // the traceback's skip speculation: deeper where a chunk has many
+        // siblings (long runs of skipped siblings), i.e. where the size-biased
+        // mean fan-out sum c^2 / sum c over the chunks' child counts c is large
+        std::vector<int64_t> nch(n, 0);
+        for (int32_t v = 0; v < n; ++v)
+            if (parent[v] >= 0) nch[parent[v]] += 1;
+        int64_t s1 = 0, s2 = 0;
+        for (int32_t v = 0; v < n; ++v) {
+            s1 += nch[v];
+            s2 += nch[v] * nch[v];
+        }
+        inst->trace_skips = s1 > 0 && s2 > 5 * s1 ? 3 : 1;
+    }
     if (!build_row_meta(n, inst->h_next, inst->h_meta, &inst->stack_depth, &inst->h_wpre, &inst->h_wave))
         return fail(PP_EINVAL, "skip-row stack deeper than supported");
     inst->h_budget.assign(budget, budget + W);

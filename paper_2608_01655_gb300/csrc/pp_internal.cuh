@@ -127,6 +127,7 @@ struct pp_instance {
     int32_t stack_depth = 0;            // skip-row stack levels needed by the DP
     int64_t total_weight = 0;           // sum of chunk weights
     int32_t max_weight = 1;             // largest chunk weight
+    int32_t trace_skips = 1;            // skips the traceback speculates per step beyond the first
     std::vector<int32_t> h_order, h_next, h_budget, h_wpre, h_meta, h_wave;
     // device tables, preorder-indexed unless noted
     int32_t *d_order = nullptr;         // [n] position -> node id
