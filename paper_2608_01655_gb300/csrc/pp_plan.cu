@@ -159,7 +159,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
                 return s;
             if ((s = mark())) return s;
             if ((s = mark())) return s;   // no traceback for the standalone scores
-            launches += 3;
+            launches += 3 + (gw.split ? 1 : 0);     // a split DP is two launches
             dp_launches += 1;
             std::vector<int64_t> score(W);
             standalone_cells = (int64_t)n * sumk;
@@ -249,7 +249,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         a.greedy = greedy;
         if ((r = launch_traceback(inst, S, work, g, kb, nullptr, &a, st))) return r;
         if ((r = mark())) return r;
-        launches += 4;
+        launches += 4 + (g.split ? 1 : 0);
         dp_launches += 1;
         return PP_OK;
     };

@@ -116,7 +116,7 @@ pp_status safeguards_impl(pp_instance *inst, cudaStream_t st, const uint32_t **m
         if ((s = launch_traceback(inst, B, wB, gB, kb, nullptr, &acc, st))) return s;
         k_or_rows<<<dim3(bx, 2), 256, 0, st>>>(n, W, 2, rows, cand);
         PP_CUDA(cudaGetLastError());
-        nl += 5;
+        nl += 5 + (gB.split ? 1 : 0);             // a split DP is two launches
         // LocalDedup: worker m sees the chunks of workers 0..m-1 in cand[2]
         uint32_t *dd = cand + 2 * N;
         for (int m = 0; m < W; ++m) {
