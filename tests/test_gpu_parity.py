@@ -438,6 +438,49 @@ def test_split_launch_matches_single_launch(pp, oracle_lib, B):
         np.testing.assert_array_equal(outs[0][2][b], och)
 
 
+def test_batch_of_16_with_stack_spill(pp, oracle_lib):
+    """A 16-item batch on a tree whose skip-row stack is deeper than shared
+    memory holds: the automatic shape (with these shared-memory needs, one
+    CTA per SM, so clusters narrower than 8 rather than a split) and a forced
+    8-CTA shape both spill stack levels to scratch; results equal each other
+    and the oracle."""
+    rng = np.random.default_rng(4242)
+    parent = [-1]
+    spine = 0
+    for _ in range(70):                 # a spine whose nodes also have a leaf child: stack ~70 deep
+        nxt = len(parent)
+        parent.append(spine)
+        parent.append(spine)
+        spine = nxt
+    for _ in range(4000):
+        parent.append(int(rng.integers(len(parent))))
+    parent = np.asarray(parent, np.int32)
+    n = len(parent)
+    weight = np.ones(n, np.int32)
+    B, k = 16, 4096
+    ppi = _tree_instance(pp, parent, weight)
+    order, nxt, depth = ppi.preorder()
+    geo = pp.pp_dp_geometry(ppi, B, k)
+    assert geo["stack_levels_smem"] < depth, (geo, depth)
+    profits = rng.integers(0, 1000, size=(B, n)).astype(np.int64)
+    profits[:, rng.random(n) < 0.3] = 0
+    budgets = rng.integers(k // 2, k + 1, size=B).astype(np.int32)
+    outs = []
+    for tune in [(0, 0), (8, 4)]:
+        pp.pp_tune_dp(*tune, False, False)
+        try:
+            outs.append(_dp_batch(pp, ppi, profits, budgets, k))
+        finally:
+            pp.pp_tune_dp(0, 0, False, False)
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
+    np.testing.assert_array_equal(outs[0][1], outs[1][1])
+    for b in (0, 7, 15):
+        ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+        assert int(outs[0][0][b]) == ob
+        np.testing.assert_array_equal(outs[0][1][b], oc)
+    ppi.close()
+
+
 def test_plan_paper_scale_properties(pp, oracle_lib):
     """The n=50,000 / 16-worker / 16-start plan the benchmark times: every
     target prefix-complete and within budget, objective equal to the oracle's
