@@ -37,6 +37,9 @@ import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
+# hardware queues for the plan's per-start streams; acts when the CUDA context
+# is created, so it is set before torch touches the GPU
+os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
 
 METRIC = "tree-DP cell-updates/s and end-to-end plan time (n=50k, 16 workers) vs HBM roofline"
 UNIT = "cell-updates/s"
@@ -407,11 +410,14 @@ def run_native(args):
     traffic = None
     if tr and tr.get("cells_swept_per_launch"):
         traffic = tr["bytes_per_launch"] * cells_swept / tr["cells_swept_per_launch"]
+    per_start = res.schedule == 2
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": alu_peak / 1e12, "unit": "Tcell/s",
                 "frac": achieved / alu_peak, "traffic": traffic,
                 "peak_source": f"derived: {SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 ALU lanes x "
                                f"{sm_mhz:.0f} MHz / {ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
-                "kernel": "k_prune + k_tree_dp_wave (one batched tree-DP launch of the plan)",
+                "kernel": ("k_prune + k_tree_dp_wave (one tree-DP step of the plan: every start's DP on its "
+                           "own stream, concurrently; duration = mean over starts of the start's DP events)"
+                           if per_start else "k_prune + k_tree_dp_wave (one batched tree-DP launch of the plan)"),
                 "launches": nl * args.steps, "launch_ms": 1000 * dp_t, "items_per_launch": items,
                 "cells_per_launch": cells_launch, "cells_swept_per_launch": cells_swept,
                 "rows_swept_per_launch": rows_swept,
@@ -480,6 +486,7 @@ def run_native(args):
             "gpu_launches": launches_per_plan * args.steps,
             "clocks": clocks,
             "plan": {"objective": best_obj, "best_start": best_start,
+                     "schedule": "per-start streams" if per_start else "lock step",
                      "dp_count": res.dp_count, "dp_cells": cells_per_plan,
                      "dp_launches": nl, "dp_rows_swept": res.dp_rows_swept,
                      "dp_cells_swept": res.dp_rows_swept * k,
@@ -488,7 +495,9 @@ def run_native(args):
             "phase_ms": {"marginals": phase_sum[0] / args.steps, "tree_dp": phase_sum[1] / args.steps,
                          "traceback_accept": phase_sum[2] / args.steps},
             "update_ms": sum(phase_sum) / (nl * args.steps),
-            "update_note": "one batched worker update (marginals + tree DP + traceback/accept) of all starts",
+            "update_note": ("one worker update (marginals + tree DP + traceback/accept) of every start, "
+                            "the starts on their own streams (phase times: mean over starts)" if per_start else
+                            "one batched worker update (marginals + tree DP + traceback/accept) of all starts"),
             "probes": probes,
             "next_steps": extras,
             "dp_geometry": {**pp.pp_dp_geometry(ppi, S, k), "split": pp.pp_dp_split(ppi, S, k)},

@@ -72,8 +72,11 @@ typedef struct {
     int32_t time_phases;           /* in: nonzero = time the phases below with CUDA events */
     float phase_ms[3];             /* out (if time_phases): device time of the marginal,
                                       tree-DP (with its row pruning) and traceback launches,
-                                      summed over the plan */
-    int32_t dp_launches;           /* out: batched tree-DP launches (one per plan step) */
+                                      summed over the plan's steps (per-start streams: the
+                                      mean over starts of each start's sum) */
+    int32_t dp_launches;           /* out: tree-DP steps (lock step: batched launches; per-start
+                                      streams: the mean over starts of executed updates),
+                                      the standalone-score launch included */
     int32_t no_safeguards;         /* in: nonzero = leave out the safeguard candidates */
     int64_t safeguard_objective[3];/* out: Independent, Popularity, LocalDedup objectives
                                       (requester-side only; else 0) */
@@ -81,6 +84,14 @@ typedef struct {
                                       chunk's holders, 2 keep top-2 holder tables per start
                                       (Section IV-C); results are identical */
     int32_t used_top2;             /* out: 1 if the top-2 tables were used */
+    int32_t schedule;              /* in: 0 automatic, 1 lock step (all starts advance together,
+                                      one batched launch per step), 2 per-start streams (each
+                                      start on its own stream, never waiting for a slower
+                                      one).  Automatic takes per-start streams when S > 1 and
+                                      CUDA_DEVICE_MAX_CONNECTIONS (read at the call; it acts
+                                      when the CUDA context is created) gives every stream its
+                                      own hardware queue, min(S, 32), else lock step.
+                                      out: the schedule used (1 or 2).  Results are identical */
 } pp_plan_stats;
 
 /*
@@ -279,7 +290,7 @@ pp_status pp_objective(pp_instance *inst, int32_t batch, const uint8_t *chosen, 
  * pp_plan_run -- Algorithm 1 (procedure PrefixPlace): for each start order,
  * one WorkerGreedy pass (Theorem 3), then at most max_rounds refinement
  * sweeps; a sweep with no accepted update ends that start.  Starts run
- * batched.  With the requester-side objective the Independent, Popularity
+ * batched in lock step, or each on its own stream (stats->schedule).  With the requester-side objective the Independent, Popularity
  * and LocalDedup placements (pp_safeguards) join the candidates as indices
  * S, S+1, S+2 unless stats->no_safeguards is set.
  *   n_starts      S >= 1

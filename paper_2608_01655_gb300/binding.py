@@ -14,6 +14,13 @@ from dataclasses import dataclass
 
 import numpy as np
 
+# The plan's per-start schedule puts each start on its own CUDA stream; the
+# driver maps streams onto CUDA_DEVICE_MAX_CONNECTIONS hardware queues (8 by
+# default), and streams sharing a queue wait on one another's launches.  The
+# variable acts when the CUDA context is created, so it is set here, before
+# that, unless the caller has chosen a value.
+os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
+
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libprefixplace.so")
 
@@ -45,7 +52,8 @@ class PlanStats(ctypes.Structure):
                 ("orders_used", _P), ("best_start", _i32), ("dp_count", _i32), ("dp_cells", _i64),
                 ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
                 ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32), ("no_safeguards", _i32),
-                ("safeguard_objective", ctypes.c_int64 * 3), ("marginals", _i32), ("used_top2", _i32)]
+                ("safeguard_objective", ctypes.c_int64 * 3), ("marginals", _i32), ("used_top2", _i32),
+                ("schedule", _i32)]
 
 
 _SIGS = {
@@ -245,11 +253,15 @@ class PlanResult:
     dp_launches: int = 0
     safeguard_objective: tuple = ()     # Independent, Popularity, LocalDedup (requester-side)
     used_top2: bool = False             # source-dependent marginals from top-2 holder tables
+    schedule: int = 0                   # 1 lock step, 2 per-start streams
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
-                time_phases: bool = False, safeguards: bool = True, marginals: int = 0) -> PlanResult:
-    """marginals (source-dependent): 0 automatic, 1 holder scan, 2 top-2 tables."""
+                time_phases: bool = False, safeguards: bool = True, marginals: int = 0,
+                schedule: int = 0) -> PlanResult:
+    """marginals (source-dependent): 0 automatic, 1 holder scan, 2 top-2 tables.
+    schedule: 0 automatic, 1 lock step (one batched launch per step), 2 one
+    stream per start; the results are identical."""
     S, W, n = int(n_starts), inst.W, inst.n
     placement = np.zeros((W, max(n, 1)), np.uint8)
     obj = _i64(0)
@@ -261,6 +273,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                    int(bool(time_phases)))
     st.no_safeguards = int(not safeguards)
     st.marginals = int(marginals)
+    st.schedule = int(schedule)
     op = None
     if orders is not None:
         orders = _np(orders, np.int32)
@@ -274,7 +287,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                       tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept),
                       int(st.dp_launches),
                       tuple(int(x) for x in st.safeguard_objective) if safeguards and inst.mode == 0 else (),
-                      bool(st.used_top2))
+                      bool(st.used_top2), int(st.schedule))
 
 
 def pp_test_inject(kind: int, value: int):

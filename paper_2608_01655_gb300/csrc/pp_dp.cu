@@ -1160,6 +1160,22 @@ DpWork dp_work_split(void *base, int batch, int n, int words)
     return w;
 }
 
+DpWork dp_work_item(const DpWork &w, int item, int n, int words)
+{
+    const size_t nb = (size_t)(n + 31) / 32 * 32, N = (size_t)std::max(n, 1), it = (size_t)item;
+    DpWork o;
+    o.bits = w.bits + it * nb * words;
+    o.rowlist = w.rowlist + it * N;
+    o.kidx = w.kidx + it * N;
+    o.cnt = w.cnt + it * (N + 1);
+    o.nkept = w.nkept + it;
+    o.skip = w.skip + it * N;
+    o.wsuf = w.wsuf + it * (N + 1);
+    o.rowp = w.rowp + it * N;
+    o.rowm = w.rowm + it * N;
+    return o;
+}
+
 // ===========================================================================
 // geometry and launch
 // ===========================================================================
@@ -1495,10 +1511,17 @@ static int dp_global_levels(const pp_instance *inst, const DpGeom &g)
     return std::max(0, inst->stack_depth - (g.split ? std::min(g.L_smem, g.L_smem2) : g.L_smem));
 }
 
+pp_status ensure_dp_stack(pp_instance *inst, const DpGeom &g, int items)
+{
+    const int L_glob = dp_global_levels(inst, g);
+    if (L_glob <= 0) return PP_OK;
+    return ensure_scratch(inst->stack, (size_t)items * L_glob * (size_t)g.kpad * sizeof(int64_t));
+}
+
 pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool by_node,
                          const int32_t *item_budget, const int32_t *item_active, const DpGeom &g,
                          int64_t *best, const DpWork &work, cudaStream_t st, int32_t max_budget,
-                         unsigned long long *rows_kept)
+                         unsigned long long *rows_kept, int stack_item)
 {
     if (batch <= 0) return PP_OK;
     if (inst->n == 0) {
@@ -1506,12 +1529,12 @@ pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bo
         return PP_OK;
     }
     const int L_glob = dp_global_levels(inst, g);
-    if (L_glob > 0) {
-        pp_status s = ensure_scratch(inst->stack, (size_t)batch * L_glob * (size_t)g.kpad * sizeof(int64_t));
-        if (s != PP_OK) return s;
-    }
+    pp_status s = ensure_dp_stack(inst, g, stack_item + batch);
+    if (s != PP_OK) return s;
+    int64_t *gstack = reinterpret_cast<int64_t *>(inst->stack.ptr);
+    if (gstack && L_glob > 0) gstack += (size_t)stack_item * L_glob * (size_t)g.kpad;
     return launch_dp_kernels(inst, batch, profit, by_node, item_budget, item_active, g, best, work, st,
-                             max_budget, reinterpret_cast<int64_t *>(inst->stack.ptr), L_glob, rows_kept);
+                             max_budget, gstack, L_glob, rows_kept);
 }
 
 pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, const DpGeom &g,

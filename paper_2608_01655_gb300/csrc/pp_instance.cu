@@ -239,6 +239,10 @@ extern "C" pp_status pp_instance_destroy(pp_instance *inst)
     if (inst->split_fork) cudaEventDestroy(inst->split_fork);
     if (inst->split_join_hi) cudaEventDestroy(inst->split_join_hi);
     if (inst->split_join_lo) cudaEventDestroy(inst->split_join_lo);
+    for (cudaStream_t x : inst->plan_streams) cudaStreamDestroy(x);
+    for (cudaEvent_t x : inst->plan_join) cudaEventDestroy(x);
+    if (inst->plan_fork) cudaEventDestroy(inst->plan_fork);
+    for (cudaEvent_t x : inst->phase_events) cudaEventDestroy(x);
     cudaSetDevice(cur);
     delete inst;
     return PP_OK;

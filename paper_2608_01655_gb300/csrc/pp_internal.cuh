@@ -107,6 +107,8 @@ struct DpWork {
 };
 size_t dp_work_bytes(int batch, int n, int words);
 DpWork dp_work_split(void *base, int batch, int n, int words);
+// the same workspace seen as a batch of one: item `item` of `w`
+DpWork dp_work_item(const DpWork &w, int item, int n, int words);
 
 // Status word values written by kernels (same numbering as pp_status).
 constexpr int32_t kDevOk = PP_OK;
@@ -155,6 +157,12 @@ struct pp_instance {
     // lower priority), forked from and joined back to the caller's stream
     cudaStream_t split_hi = nullptr, split_lo = nullptr;
     cudaEvent_t split_fork = nullptr, split_join_hi = nullptr, split_join_lo = nullptr;
+    // pp_plan_run without lock step: one stream per start (up to kPlanStreams),
+    // forked from and joined back to the caller's stream
+    std::vector<cudaStream_t> plan_streams;
+    std::vector<cudaEvent_t> plan_join;
+    cudaEvent_t plan_fork = nullptr;
+    std::vector<cudaEvent_t> phase_events;      // timing events of pp_plan_run, reused across calls
 };
 
 namespace pp {
@@ -178,10 +186,14 @@ bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int bat
 // Launchers used by both the ABI calls and the planner.
 //   prof_by_node: profits indexed by node id (ABI) instead of preorder
 //   item_budget:  [batch] budgets; item_active: [batch] or null (0 = skip item)
+// stack_item: the launch's items use skip-row stack scratch from item slot
+// stack_item on (launches of disjoint slots may run concurrently)
 pp_status launch_tree_dp(pp_instance *inst, int batch, const int64_t *profit, bool prof_by_node,
                          const int32_t *item_budget, const int32_t *item_active,
                          const DpGeom &g, int64_t *best, const DpWork &work, cudaStream_t st,
-                         int32_t max_budget, unsigned long long *rows_kept = nullptr);
+                         int32_t max_budget, unsigned long long *rows_kept = nullptr, int stack_item = 0);
+// scratch for the skip-row stack of `items` item slots of geometry g
+pp_status ensure_dp_stack(pp_instance *inst, const DpGeom &g, int items);
 
 pp_status launch_marginals(pp_instance *inst, int batch, const int32_t *worker,
                            const uint32_t *mask, bool by_node, const int32_t *item_active,

@@ -7,6 +7,7 @@
 // (its later kernels return at once).  Holder sets live on the device as one
 // 32-bit mask per chunk and start, in preorder.
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <numeric>
 
@@ -19,13 +20,40 @@ namespace pp {
 constexpr size_t kTop2MaxBytes = (size_t)16 << 30;
 
 // per-sweep bookkeeping: a start that accepted nothing is done
-__global__ void k_sweep_end(int S, int32_t *active, const int32_t *improved, int32_t *sweeps)
+__global__ void k_sweep_end(int S, int32_t *active, int32_t *improved, int32_t *sweeps)
 {
     int s = blockIdx.x * blockDim.x + threadIdx.x;
     if (s < S && active[s]) {
         sweeps[s] += 1;
         active[s] = improved[s];
+        improved[s] = 0;                // for the next sweep
     }
+}
+
+// streams of the per-start schedule (starts beyond share them round-robin)
+constexpr int kPlanStreams = 32;
+
+static pp_status ensure_plan_streams(pp_instance *inst, int ns)
+{
+    while ((int)inst->plan_streams.size() < ns) {
+        cudaStream_t x;
+        cudaEvent_t e;
+        PP_CUDA(cudaStreamCreateWithFlags(&x, cudaStreamNonBlocking));
+        inst->plan_streams.push_back(x);
+        PP_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+        inst->plan_join.push_back(e);
+    }
+    if (!inst->plan_fork) PP_CUDA(cudaEventCreateWithFlags(&inst->plan_fork, cudaEventDisableTiming));
+    return PP_OK;
+}
+
+// CUDA_DEVICE_MAX_CONNECTIONS as the process sees it now (8 when unset); the
+// driver reads it when the context is created
+static int hardware_queues()
+{
+    const char *e = std::getenv("CUDA_DEVICE_MAX_CONNECTIONS");
+    const int c = e ? std::atoi(e) : 8;
+    return c > 0 ? c : 8;
 }
 
 // SplitMix64 (Steele, Lea and Flood, OOPSLA 2014)
@@ -89,6 +117,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
                     cudaStream_t st, bool orders_only)
 {
     const int32_t n = inst->n, W = inst->W;
+    if (stats && (stats->schedule < 0 || stats->schedule > 2)) return fail(PP_EINVAL, "schedule must be 0, 1 or 2");
     int launches = 0;
     int64_t standalone_cells = 0;
     int32_t maxk = 0;
@@ -115,15 +144,23 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
     // optional per-phase timing: events around every launch, read once at the end
     const bool timing = stats && stats->time_phases;
     int32_t dp_launches = 0;
-    struct Events {
-        std::vector<cudaEvent_t> v;
-        ~Events() { for (cudaEvent_t e : v) cudaEventDestroy(e); }
-    } ev;
+    std::vector<cudaEvent_t> ev;        // lock step: every mark; per-start streams: the standalone step
+    size_t pool_used = 0;
+    auto take = [&](cudaEvent_t *e) -> pp_status {
+        if (pool_used == inst->phase_events.size()) {
+            cudaEvent_t x;
+            PP_CUDA(cudaEventCreate(&x));
+            inst->phase_events.push_back(x);
+        }
+        *e = inst->phase_events[pool_used++];
+        return PP_OK;
+    };
     auto mark = [&]() -> pp_status {
         if (!timing) return PP_OK;
         cudaEvent_t e;
-        PP_CUDA(cudaEventCreate(&e));
-        ev.v.push_back(e);
+        pp_status r = take(&e);
+        if (r) return r;
+        ev.push_back(e);
         PP_CUDA(cudaEventRecord(e, st));
         return PP_OK;
     };
@@ -220,62 +257,151 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         PP_CUDA(cudaMemsetAsync(base, 0, b2, st));                 // v1 = v2 = 0: no holders yet
         PP_CUDA(cudaMemsetAsync(t2.l1, 0xFF, tw, st));             // l1 = -1
     }
-    const int32_t *prev_wk = nullptr;     // top-2: worker of the previous step, per start
-    auto step = [&](int t, int greedy) -> pp_status {
-        const int32_t *wk = pb.work + (size_t)t * B;
-        const int32_t *kb = pb.kbud + (size_t)t * B;
-        pp_status r;
-        if ((r = mark())) return r;
-        if (use_top2) {
-            // the previous step's change is folded into this step's marginal pass
-            r = launch_marginals_top2(inst, S, prev_wk, wk, pb.mask, pb.active, t2, pb.profit, pb.oldsum, st);
-            prev_wk = wk;
-        } else {
-            r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st);
-        }
-        if (r) return r;
-        if ((r = mark())) return r;
-        if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, work, st, maxk, rows_kept)))
-            return r;
-        if ((r = mark())) return r;
-        AcceptArgs a;
-        a.worker = wk;
-        a.best = pb.best;
-        a.oldsum = pb.oldsum;
-        a.active = pb.active;
-        a.improved = pb.improved;
-        a.accepted = pb.accepted;
-        a.mask = pb.mask;
-        a.greedy = greedy;
-        if ((r = launch_traceback(inst, S, work, g, kb, nullptr, &a, st))) return r;
-        if ((r = mark())) return r;
-        launches += 4 + (g.split ? 1 : 0);
-        dp_launches += 1;
-        return PP_OK;
-    };
+    PP_CUDA(cudaMemsetAsync(pb.improved, 0, 4 * S, st));
+    // lock step unless asked for per-start streams, or (automatic) unless every
+    // start's stream gets a hardware queue of its own: streams that share a
+    // queue wait on one another's launches, which costs more than lock step
+    const int32_t sched = stats ? stats->schedule : 0;
+    const bool lockstep = S == 1 || sched == 1 ||
+                          (sched == 0 && hardware_queues() < std::min<int>(S, kPlanStreams));
+    int32_t start_steps = 0;            // per-start streams: updates launched per start
+    std::vector<std::vector<cudaEvent_t>> sev;   // per-start streams: each start's phase events
+    if (lockstep) {
+        const int32_t *prev_wk = nullptr;     // top-2: worker of the previous step, per start
+        auto step = [&](int t, int greedy) -> pp_status {
+            const int32_t *wk = pb.work + (size_t)t * B;
+            const int32_t *kb = pb.kbud + (size_t)t * B;
+            pp_status r;
+            if ((r = mark())) return r;
+            if (use_top2) {
+                // the previous step's change is folded into this step's marginal pass
+                r = launch_marginals_top2(inst, S, prev_wk, wk, pb.mask, pb.active, t2, pb.profit, pb.oldsum, st);
+                prev_wk = wk;
+            } else {
+                r = launch_marginals(inst, S, wk, pb.mask, false, pb.active, pb.profit, pb.oldsum, st);
+            }
+            if (r) return r;
+            if ((r = mark())) return r;
+            if ((r = launch_tree_dp(inst, S, pb.profit, false, kb, pb.active, g, pb.best, work, st, maxk, rows_kept)))
+                return r;
+            if ((r = mark())) return r;
+            AcceptArgs a;
+            a.worker = wk;
+            a.best = pb.best;
+            a.oldsum = pb.oldsum;
+            a.active = pb.active;
+            a.improved = pb.improved;
+            a.accepted = pb.accepted;
+            a.mask = pb.mask;
+            a.greedy = greedy;
+            if ((r = launch_traceback(inst, S, work, g, kb, nullptr, &a, st))) return r;
+            if ((r = mark())) return r;
+            launches += 4 + (g.split ? 1 : 0);
+            dp_launches += 1;
+            return PP_OK;
+        };
 
-    // WorkerGreedy pass
-    for (int32_t t = 0; t < W; ++t)
-        if ((s = step(t, 1))) return s;
-    dp_count += S * W;
-    cells += (int64_t)S * n * sumk;
-
-    // coordinate refinement
-    std::vector<int32_t> act(S, 1);
-    for (int32_t r = 0; r < R; ++r) {
-        int nact = 0;
-        for (int32_t x = 0; x < S; ++x) nact += act[x] != 0;
-        if (nact == 0) break;
-        PP_CUDA(cudaMemsetAsync(pb.improved, 0, 4 * S, st));
+        // WorkerGreedy pass
         for (int32_t t = 0; t < W; ++t)
-            if ((s = step(t, 0))) return s;
-        dp_count += nact * W;
-        cells += (int64_t)nact * n * sumk;
-        k_sweep_end<<<(S + 127) / 128, 128, 0, st>>>(S, pb.active, pb.improved, pb.sweeps);
-        PP_CUDA(cudaGetLastError());
-        launches += 1;
-        PP_CUDA(cudaMemcpyAsync(act.data(), pb.active, 4 * S, cudaMemcpyDeviceToHost, st));
-        PP_CUDA(cudaStreamSynchronize(st));
+            if ((s = step(t, 1))) return s;
+        dp_count += S * W;
+        cells += (int64_t)S * n * sumk;
+
+        // coordinate refinement
+        std::vector<int32_t> act(S, 1);
+        for (int32_t r = 0; r < R; ++r) {
+            int nact = 0;
+            for (int32_t x = 0; x < S; ++x) nact += act[x] != 0;
+            if (nact == 0) break;
+            PP_CUDA(cudaMemsetAsync(pb.improved, 0, 4 * S, st));
+            for (int32_t t = 0; t < W; ++t)
+                if ((s = step(t, 0))) return s;
+            dp_count += nact * W;
+            cells += (int64_t)nact * n * sumk;
+            k_sweep_end<<<(S + 127) / 128, 128, 0, st>>>(S, pb.active, pb.improved, pb.sweeps);
+            PP_CUDA(cudaGetLastError());
+            launches += 1;
+            PP_CUDA(cudaMemcpyAsync(act.data(), pb.active, 4 * S, cudaMemcpyDeviceToHost, st));
+            PP_CUDA(cudaStreamSynchronize(st));
+        }
+    } else {
+        // Every start on its own stream: start s runs its W (1 + R) updates
+        // back to back and never waits for a slower start (in lock step each
+        // step waits for the start with the most kept rows).  Each update is
+        // the same kernels at batch one on the start's slice of every buffer,
+        // in the batch's launch shape (no split: a launch holds one item).
+        // All R sweeps are enqueued; a start whose sweep accepted nothing is
+        // inactive from then on and its later kernels return at once.
+        const int NS = std::min(S, kPlanStreams);
+        if ((s = ensure_plan_streams(inst, NS))) return s;
+        if ((s = ensure_dp_stack(inst, g, S))) return s;   // one stack slot per start, allocated up front
+        DpGeom g1 = g;
+        g1.split = 0;
+        PP_CUDA(cudaEventRecord(inst->plan_fork, st));
+        for (int x = 0; x < NS; ++x) PP_CUDA(cudaStreamWaitEvent(inst->plan_streams[x], inst->plan_fork, 0));
+        std::vector<const int32_t *> prev(S, nullptr);
+        sev.resize(timing ? S : 0);
+        auto smark = [&](int x, cudaStream_t sx) -> pp_status {
+            if (!timing) return PP_OK;
+            cudaEvent_t e;
+            pp_status r = take(&e);
+            if (r) return r;
+            sev[x].push_back(e);
+            PP_CUDA(cudaEventRecord(e, sx));
+            return PP_OK;
+        };
+        const size_t N = (size_t)std::max(n, 1);
+        for (int q = 0; q < W * (1 + R); ++q) {
+            const int pass = q / W, t = q % W;
+            for (int x = 0; x < S; ++x) {
+                cudaStream_t sx = inst->plan_streams[x % NS];
+                const int32_t *wk = pb.work + (size_t)t * B + x;
+                const int32_t *kb = pb.kbud + (size_t)t * B + x;
+                uint32_t *mk = pb.mask + (size_t)x * N;
+                int64_t *pf = pb.profit + (size_t)x * N;
+                if ((s = smark(x, sx))) return s;
+                if (use_top2) {
+                    Top2 tx = t2;
+                    tx.v1 += (size_t)x * W * N;
+                    tx.v2 += (size_t)x * W * N;
+                    tx.l1 += (size_t)x * W * N;
+                    tx.oldbit += (size_t)x * N;
+                    s = launch_marginals_top2(inst, 1, prev[x], wk, mk, pb.active + x, tx, pf, pb.oldsum + x, sx);
+                    prev[x] = wk;
+                } else {
+                    s = launch_marginals(inst, 1, wk, mk, false, pb.active + x, pf, pb.oldsum + x, sx);
+                }
+                if (s) return s;
+                if ((s = smark(x, sx))) return s;
+                const DpWork wx = dp_work_item(work, x, n, g.words);
+                if ((s = launch_tree_dp(inst, 1, pf, false, kb, pb.active + x, g1, pb.best + x, wx, sx, maxk,
+                                        rows_kept, x)))
+                    return s;
+                if ((s = smark(x, sx))) return s;
+                AcceptArgs a;
+                a.worker = wk;
+                a.best = pb.best + x;
+                a.oldsum = pb.oldsum + x;
+                a.active = pb.active + x;
+                a.improved = pb.improved + x;
+                a.accepted = pb.accepted + x;
+                a.mask = mk;
+                a.greedy = pass == 0;
+                if ((s = launch_traceback(inst, 1, wx, g1, kb, nullptr, &a, sx))) return s;
+                if ((s = smark(x, sx))) return s;
+                launches += 4;
+                if (pass > 0 && t == W - 1) {
+                    k_sweep_end<<<1, 32, 0, sx>>>(1, pb.active + x, pb.improved + x, pb.sweeps + x);
+                    PP_CUDA(cudaGetLastError());
+                    launches += 1;
+                }
+            }
+        }
+        start_steps = W * (1 + R);
+        for (int x = 0; x < NS; ++x) {
+            PP_CUDA(cudaEventRecord(inst->plan_join[x], inst->plan_streams[x]));
+            PP_CUDA(cudaStreamWaitEvent(st, inst->plan_join[x], 0));
+        }
     }
 
     // objective of every candidate, argmax (ties to the lowest start)
@@ -289,6 +415,14 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
     PP_CUDA(cudaMemcpyAsync(sw.data(), pb.sweeps, 4 * S, cudaMemcpyDeviceToHost, st));
     PP_CUDA(cudaMemcpyAsync(acc.data(), pb.accepted, 4 * S, cudaMemcpyDeviceToHost, st));
     PP_CUDA(cudaStreamSynchronize(st));
+    if (!lockstep) {
+        // executed updates, from the sweeps each start ran (the greedy pass always runs)
+        int64_t swsum = 0;
+        for (int32_t x = 0; x < S; ++x) swsum += sw[x];
+        dp_count += (int)(S * W + swsum * W);
+        cells += ((int64_t)S + swsum) * n * sumk;
+        dp_launches += (int32_t)((W * (S + swsum) + S / 2) / S);
+    }
     int32_t bs = 0;
     for (int32_t x = 1; x < S; ++x)
         if (obj[x] > obj[bs]) bs = x;
@@ -335,15 +469,27 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         stats->dp_launches = dp_launches;
         for (int c = 0; c < 3; ++c) stats->safeguard_objective[c] = so[c];
         stats->used_top2 = use_top2;
+        stats->schedule = lockstep ? 1 : 2;
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
-        for (size_t x = 0; x + 3 < ev.v.size(); x += 4) {
-            float a = 0.f, b = 0.f, c = 0.f;
-            cudaEventElapsedTime(&a, ev.v[x], ev.v[x + 1]);
-            cudaEventElapsedTime(&b, ev.v[x + 1], ev.v[x + 2]);
-            cudaEventElapsedTime(&c, ev.v[x + 2], ev.v[x + 3]);
-            stats->phase_ms[0] += a;
-            stats->phase_ms[1] += b;
-            stats->phase_ms[2] += c;
+        // groups of four marks: before the marginals, the DP and the traceback, and after
+        auto add = [&](const std::vector<cudaEvent_t> &v, size_t from, size_t to, float scale) {
+            to = std::min(to, v.size());       // no events without time_phases
+            for (size_t x = from; x + 3 < to; x += 4) {
+                float a = 0.f, b = 0.f, c = 0.f;
+                cudaEventElapsedTime(&a, v[x], v[x + 1]);
+                cudaEventElapsedTime(&b, v[x + 1], v[x + 2]);
+                cudaEventElapsedTime(&c, v[x + 2], v[x + 3]);
+                stats->phase_ms[0] += a * scale;
+                stats->phase_ms[1] += b * scale;
+                stats->phase_ms[2] += c * scale;
+            }
+        };
+        if (lockstep) {
+            add(ev, 0, ev.size(), 1.f);
+        } else {
+            // the standalone-score step (on the caller's stream), then the mean over starts
+            add(ev, 0, standalone_cells ? 4 : 0, 1.f);
+            for (const auto &v : sev) add(v, 0, v.size(), 1.f / (float)S);
         }
     }
     return PP_OK;

@@ -3,6 +3,10 @@ import sys
 
 import pytest
 
+# hardware queues for the plan's per-start streams; acts when the CUDA
+# context is created, so it is set before any test touches the GPU
+os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
+
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)

@@ -481,6 +481,26 @@ def test_batch_of_16_with_stack_spill(pp, oracle_lib):
     ppi.close()
 
 
+@pytest.mark.parametrize("cfg", [1, 2])
+def test_plan_per_start_streams_match_lockstep(pp, cfg):
+    """The per-start-stream schedule (each start on its own stream, never
+    waiting for a slower one) and the lock-step schedule (one batched launch
+    per step) give the same plan, statistics included."""
+    inst = wl.make(cfg)
+    with pp.Instance.from_workload(inst) as ppi:
+        a = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds, schedule=2)
+        b = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds, schedule=1)
+        with pytest.raises(pp.PPError):
+            pp.pp_plan_run(ppi, inst.starts, None, inst.rounds, schedule=3)
+    assert (a.schedule, b.schedule) == (2, 1)
+    assert a.objective == b.objective and a.best_start == b.best_start
+    np.testing.assert_array_equal(a.placement, b.placement)
+    np.testing.assert_array_equal(a.per_start_objective, b.per_start_objective)
+    np.testing.assert_array_equal(a.per_start_sweeps, b.per_start_sweeps)
+    np.testing.assert_array_equal(a.per_start_accepted, b.per_start_accepted)
+    assert (a.dp_count, a.dp_cells, a.dp_rows_swept) == (b.dp_count, b.dp_cells, b.dp_rows_swept)
+
+
 def test_plan_paper_scale_properties(pp, oracle_lib):
     """The n=50,000 / 16-worker / 16-start plan the benchmark times: every
     target prefix-complete and within budget, objective equal to the oracle's
