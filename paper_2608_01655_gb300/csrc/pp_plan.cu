@@ -337,6 +337,15 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         if ((s = ensure_dp_stack(inst, g, S))) return s;   // one stack slot per start, allocated up front
         DpGeom g1 = g;
         g1.split = 0;
+        {
+            // more than half an SM's shared memory per CTA: two DP CTAs on one SM
+            // slow each other down (~25% per row); with one per SM a start whose
+            // cluster finds no room waits instead (plan 208.6 -> 205.6 ms)
+            int per_sm = 0, optin = 0;
+            PP_CUDA(cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, inst->device));
+            PP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, inst->device));
+            g1.smem = std::max(g1.smem, (size_t)std::min(per_sm / 2, optin));
+        }
         PP_CUDA(cudaEventRecord(inst->plan_fork, st));
         for (int x = 0; x < NS; ++x) PP_CUDA(cudaStreamWaitEvent(inst->plan_streams[x], inst->plan_fork, 0));
         std::vector<const int32_t *> prev(S, nullptr);
