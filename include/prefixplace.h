@@ -47,7 +47,7 @@ typedef enum {
     PP_OK = 0,
     PP_EINVAL = 1,      /* bad argument: size, mode, null pointer, weight < 1, negative data */
     PP_ENOTTREE = 2,    /* parent[] out of range, self-parent, or a cycle */
-    PP_EOVERFLOW = 3,   /* sum_b sum_m demand * recompute exceeds 2^62 */
+    PP_EOVERFLOW = 3,   /* sum of demand * recompute, of demand or of recompute exceeds 2^62 */
     PP_ENOMEM = 4,      /* device or host allocation failed */
     PP_ECUDA = 5,       /* a CUDA runtime call failed */
     PP_ETIMEOUT = 6,    /* a bounded device-side wait ran out (device status word) */
@@ -114,9 +114,11 @@ typedef struct {
  *   budget        host [W]: k_m >= 0 slots
  *   stream        stream for the uploads and precompute kernels
  *   out           receives the instance (NULL on failure)
- * Errors: PP_EINVAL, PP_ENOTTREE, PP_EOVERFLOW (sum_b sum_m Lambda * w,
- * computed exactly, above 2^62; this bound keeps every objective, marginal
- * and DP value of the instance inside int64), PP_ENOMEM, PP_ECUDA.
+ * Errors: PP_EINVAL, PP_ENOTTREE, PP_EOVERFLOW (one of three exact sums
+ * over all (m, b) above 2^62: Lambda * w, which bounds every objective,
+ * marginal and DP value of the planner; Lambda, which bounds the Popularity
+ * safeguard's DP values; w, which bounds the epoch update's one-time cost),
+ * PP_ENOMEM, PP_ECUDA.
  * The call synchronises `stream` before returning; the inputs are not retained.
  */
 pp_status pp_instance_create(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
@@ -399,7 +401,8 @@ typedef struct {
     int64_t incumbent_objective;   /* G(T_old) under the instance's (refreshed) demand */
     int64_t new_objective;         /* G(T_new) of the reoptimised target */
     int64_t materialization_cost;  /* one-time cost of the chunks T_new adds, microseconds */
-    int64_t break_even_requests;   /* ceil(cost * epoch_requests / (G_new - G_old)); -1 without a gain */
+    int64_t break_even_requests;   /* ceil(cost * epoch_requests / (G_new - G_old)), INT64_MAX when
+                                      that does not fit in int64; -1 without a gain */
     int32_t adopted;               /* 1: T_new returned; 0: the incumbent kept */
 } pp_replan_result;
 

@@ -64,6 +64,7 @@ def _load():
             "or_safeguards": (ctypes.c_int, [P, P, P]),
             "or_replan": (ctypes.c_int, [P, P, i32, P, i32, i64, i64, i32, ctypes.c_int, P, P]),
             "or_worker_update": (i64, [P, i32, P, P, P]),
+            "or_splitmix64": (None, [ctypes.c_uint64, i32, P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(lib, name)
@@ -165,6 +166,13 @@ def standalone(prob: Problem) -> np.ndarray:
     if _load().or_standalone(prob.ref, _ptr(out)) != 0:
         raise ValueError("parent array is not a forest")
     return out
+
+
+def splitmix64(seed: int, count: int) -> np.ndarray:
+    """The first `count` outputs of the oracle's SplitMix64 from state `seed`."""
+    out = np.zeros(max(count, 1), np.uint64)
+    _load().or_splitmix64(int(seed), int(count), _ptr(out))
+    return out[:count]
 
 
 def default_orders(prob: Problem, S: int) -> np.ndarray:

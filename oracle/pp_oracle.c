@@ -205,7 +205,8 @@ void or_marginal(const or_inst *I, int32_t h, const uint8_t *placement, int64_t 
 /* The branch is recorded as "take" only when it is strictly larger, and    */
 /* the backtrack starts at (0, k).  Returns D[0][k]; chosen[] is by node id. */
 /*                                                                          */
-/* variant 0: the whole (n+1) x (k+1) table, as Algorithm 1 writes it.      */
+/* variant 0: the whole (n+1) x (k+1) table of Eq. 9 and one decision per  */
+/*            cell (Theorem 1's O(nk) time and memory).                     */
 /* variant 1: the same recurrence; a row is freed after its last reader     */
 /*            (min{i : next(i) = r or i + 1 = r}), decisions kept as bits.  */
 /* variant -1: 0 when the table is at most 64 MiB, else 1.                  */
@@ -345,6 +346,14 @@ static uint64_t splitmix64_next(uint64_t *state)
     return z ^ (z >> 31);
 }
 
+/* The first `count` outputs of SplitMix64 from state `seed` (exposed so the */
+/* tests can check the generator against its published outputs).             */
+void or_splitmix64(uint64_t seed, int32_t count, uint64_t *out)
+{
+    uint64_t st = seed;
+    for (int32_t i = 0; i < count; ++i) out[i] = splitmix64_next(&st);
+}
+
 /* Start orders (Section IV-C).  S == 1: identity.  Otherwise start 0 is     */
 /* the standalone-score order (descending, ties to the lower worker id),     */
 /* start 1 its reverse, and start s >= 2 the Fisher-Yates shuffle of the     */
@@ -378,12 +387,16 @@ int or_default_orders(const or_inst *I, int32_t S, int32_t *orders)
 }
 
 /* ------------------------------------------------------------------------ */
-/* Algorithm 1, procedure PrefixPlace, for one start order pi:              */
-/*   greedy pass: T_m <- {} for all m; for h in pi: T_h <- RootedDP(p_h, k_h) */
-/*   refinement (at most R sweeps): for h in pi: g_old <- G(T); T_h <- {};   */
-/*     T'_h <- RootedDP(p_h, k_h); accept iff G(T_{-h}, T'_h) > g_old       */
-/*     (recomputed in full, not through the additive shortcut);             */
-/*   a sweep with no accepted update ends the start.                        */
+/* One start of the planner (Section IV-C) for the worker sequence pi.       */
+/* Every target begins empty.  Greedy pass (Theorem 3): the workers of pi,   */
+/* one after another, each get the exact best prefix-complete target for    */
+/* their marginals (Eq. 10 / Eq. 7) given what the workers before them      */
+/* hold; the workers after them still hold nothing.  Refinement: at most R  */
+/* passes over pi; in a pass each worker's target is solved again against   */
+/* the others' current targets (its own is dropped first) and kept only if */
+/* the objective, evaluated from scratch on the whole placement (Eq. 4 /    */
+/* Eq. 6) right before and after, strictly grows; otherwise the old target  */
+/* comes back.  A pass that kept no new target ends the start.              */
 /* ------------------------------------------------------------------------ */
 typedef struct {
     const or_inst *I;
@@ -579,7 +592,8 @@ int32_t or_plan(const or_inst *I, int32_t S, const int32_t *orders, int32_t R, i
 /* of epoch_requests requests, so T_new is adopted iff                        */
 /*   (G(T_new) - G(T_old)) * horizon_requests > cost * epoch_requests,        */
 /* and break-even requests = ceil(cost * epoch_requests / (G_new - G_old))    */
-/* (-1 without a gain).  out5 = {G_old, G_new, cost, break_even, adopted};   */
+/* (-1 without a gain; INT64_MAX when the ceiling does not fit in int64).  */
+/* out5 = {G_old, G_new, cost, break_even, adopted};                          */
 /* placement [W][n] out = the adopted target.  Returns 0, or -1 on an        */
 /* invalid tree.                                                              */
 /* ------------------------------------------------------------------------ */
@@ -609,9 +623,10 @@ int or_replan(const or_inst *I, const uint8_t *incumbent, int32_t S, const int32
         }
     int64_t gain = g_new - g_old;
     int64_t be = -1;
-    if (gain > 0) {
+    if (gain > 0) {                     /* the ceiling, saturated at INT64_MAX */
         __int128 num = (__int128)cost * epoch_requests;
-        be = (int64_t)((num + gain - 1) / gain);
+        __int128 q = (num + gain - 1) / gain;
+        be = q > (__int128)INT64_MAX ? INT64_MAX : (int64_t)q;
     }
     int adopt = gain > 0 && (__int128)gain * horizon_requests > (__int128)cost * epoch_requests;
     memcpy(placement, adopt ? T : incumbent, (size_t)W * n);

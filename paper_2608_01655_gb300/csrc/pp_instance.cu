@@ -276,15 +276,23 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     }
     const size_t Wn = (size_t)W * n;
     const size_t tn = mode == PP_TRANSFER_SOURCE ? (size_t)W * Wn : Wn;
-    __int128 total = 0;
+    // Three exact sums bound every int64 value the library forms:
+    //  sum Lambda * w: objectives (Eq. 4, Eq. 6), marginals and DP values;
+    //  sum Lambda:     the Popularity safeguard's DP values (profit Lambda);
+    //  sum w:          the epoch update's one-time cost (at most one w per (m, b)).
+    __int128 total = 0, sum_demand = 0, sum_recompute = 0;
     for (size_t x = 0; x < Wn; ++x) {
         if (demand[x] < 0 || recompute[x] < 0) return fail(PP_EINVAL, "negative demand or recompute cost");
         total += (__int128)demand[x] * (__int128)recompute[x];
+        sum_demand += demand[x];
+        sum_recompute += recompute[x];
     }
     for (size_t x = 0; x < tn; ++x)
         if (transfer[x] < 0) return fail(PP_EINVAL, "negative transfer cost");
-    if (total > ((__int128)1 << 62))
-        return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
+    const __int128 lim = (__int128)1 << 62;
+    if (total > lim) return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
+    if (sum_demand > lim) return fail(PP_EOVERFLOW, "sum of demand exceeds 2^62");
+    if (sum_recompute > lim) return fail(PP_EOVERFLOW, "sum of recompute costs exceeds 2^62");
 
     inst->n = n;
     inst->W = W;

@@ -7,6 +7,7 @@
 // it in the incumbent (recomputing when none does).  The target is adopted iff
 //   (G(T_new) - G(T_old)) * horizon_requests > cost * epoch_requests,
 // G being a saving per epoch of epoch_requests requests.
+#include <cstdint>
 #include <cstring>
 #include <vector>
 
@@ -85,9 +86,10 @@ extern "C" pp_status pp_replan(pp_instance *inst, const uint8_t *incumbent, int3
     result->new_objective = g_new;
     result->materialization_cost = cost;
     result->break_even_requests = -1;
-    if (gain > 0) {
+    if (gain > 0) {                     // the ceiling, saturated at INT64_MAX
         const __int128 num = (__int128)cost * epoch_requests;
-        result->break_even_requests = (int64_t)((num + gain - 1) / gain);
+        const __int128 q = (num + gain - 1) / gain;
+        result->break_even_requests = q > (__int128)INT64_MAX ? INT64_MAX : (int64_t)q;
     }
     result->adopted = gain > 0 && (__int128)gain * horizon_requests > (__int128)cost * epoch_requests;
     std::memcpy(placement, result->adopted ? target.data() : incumbent, Wn);

@@ -157,3 +157,61 @@ def materialisation_cost(inst, old, new) -> int:
                 w = min(w, fetch)
             total += w
     return total
+
+
+def standalone_score(inst, h) -> int:
+    """Worker h's best Section III-A saving when it is the only holder
+    (the standalone score of Section IV-C), by enumeration."""
+    best = 0
+    for s in parent_closed_masks(inst.parent, inst.weight, int(inst.budget[h])):
+        pl = np.zeros((inst.W, inst.n), bool)
+        pl[h] = s
+        best = max(best, materialisation_saving(inst, pl))
+    return best
+
+
+def coordinate_trajectory(inst, pi, R, sweep_order=None, stale_reference=False):
+    """One start of the planner (Section IV-C) rebuilt from enumeration.
+
+    A worker update replaces T_h by the parent-closed set within k_h that
+    maximises the Section III-A saving of the whole placement with the other
+    targets fixed (ties to the lexicographically smallest preorder indicator,
+    the DP's rule); by Prop. 1 this is the set the DP of Eq. 9 finds on the
+    worker's marginals.  Greedy pass: the workers of `pi` in turn, the later
+    ones still empty.  Refinement: at most R sweeps over `pi`; a new target
+    is kept only if the saving strictly exceeds the saving just before the
+    update; a sweep that keeps nothing ends the start.
+
+    `sweep_order` and `stale_reference` only exist to build deliberately
+    wrong variants (another sweep order; comparing against the saving at the
+    start of the sweep) and show that the pins tell them apart.
+    Returns (placement [W][n] uint8, saving, sweeps, accepted)."""
+    W, n = inst.W, inst.n
+    T = np.zeros((W, n), np.uint8)
+
+    def best_for(h):
+        def value(s):
+            X = T.copy()
+            X[h] = s
+            return materialisation_saving(inst, X)
+        return best_set_by(inst.parent, inst.weight, int(inst.budget[h]), value)
+
+    for h in pi:
+        T[h] = best_for(h)
+    sweeps = accepted = 0
+    for _ in range(R):
+        sweeps += 1
+        kept = False
+        at_sweep_start = materialisation_saving(inst, T)
+        for h in (pi if sweep_order is None else sweep_order):
+            before = at_sweep_start if stale_reference else materialisation_saving(inst, T)
+            old = T[h].copy()
+            T[h] = best_for(h)
+            if materialisation_saving(inst, T) > before:
+                kept = True
+                accepted += 1
+            else:
+                T[h] = old
+        if not kept:
+            break
+    return T, materialisation_saving(inst, T), sweeps, accepted

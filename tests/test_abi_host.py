@@ -72,6 +72,19 @@ def test_create_validation_is_host_side(lib):
     big = np.full((2, 6), 1 << 30, np.int64)       # 12 products of 2^60 > 2^62
     assert _create(lib, demand=big, recompute=big) == lib.PP_EOVERFLOW
     assert "2^62" in lib.last_error()
+    # the Popularity safeguard's DP values (profit Lambda) stay bounded even
+    # where w = 0 makes every Lambda * w vanish
+    huge = np.full((2, 6), 1 << 59, np.int64)      # 12 x 2^59 > 2^62
+    assert _create(lib, demand=huge, recompute=np.zeros((2, 6), np.int64)) == lib.PP_EOVERFLOW
+    assert "sum of demand" in lib.last_error()
+    # the epoch update's one-time cost (one w per newly held (m, b)) stays
+    # bounded even where Lambda = 0
+    assert _create(lib, demand=np.zeros((2, 6), np.int64), recompute=huge) == lib.PP_EOVERFLOW
+    assert "recompute" in lib.last_error()
+    # just inside every bound: accepted up to the CUDA part of the call
+    edge = np.full((2, 6), (1 << 62) // 12, np.int64)
+    st = _create(lib, demand=edge, recompute=np.zeros((2, 6), np.int64))
+    assert st != lib.PP_EOVERFLOW
 
 
 def test_row_plan_preorder_matches_definition(lib):

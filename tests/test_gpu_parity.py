@@ -341,6 +341,26 @@ def test_replan_matches_oracle(pp, oracle_lib, mode):
                 pp.pp_replan(ppi, old, S, R, 0, 1)
 
 
+def test_replan_break_even_saturates_like_oracle(pp, oracle_lib):
+    """Break-even requests whose exact ceiling exceeds int64 saturate at
+    INT64_MAX on both sides; smaller ones stay exact."""
+    rng = np.random.default_rng(91)
+    big = 0
+    for trial in range(8):
+        inst = wl.random_small(rng, 30, 3, trial % 2, k_max=8, w_max=1, demand_max=1)
+        prob = oracle_lib.Problem.from_instance(inst)
+        old = oracle_lib.plan(prob, 1, 0, orders=np.array([[2, 1, 0]], np.int32), threads=1,
+                              safeguards=False).placement
+        epoch = (1 << 63) - 1 if trial % 3 else 30000
+        o = oracle_lib.replan(prob, old, 2, 2, epoch, 1)
+        with pp.Instance.from_workload(inst) as ppi:
+            g = pp.pp_replan(ppi, old, 2, 2, epoch, 1)
+        assert (g.new_objective, g.materialization_cost, g.break_even_requests, g.adopted) == \
+            (o.new_objective, o.materialization_cost, o.break_even_requests, o.adopted)
+        big += o.break_even_requests == (1 << 63) - 1
+    assert big >= 2
+
+
 def _random_feasible_placement(rng, inst, frac):
     """Parent-closed, within-budget placement grown top-down (a plausible
     mid-refinement state to sample one update from)."""

@@ -491,3 +491,31 @@ def test_refinement_accepts_only_strict_improvements(oracle_lib):
         else:
             assert r.per_start_accepted[0] >= 1
     assert seen >= 10
+
+
+def test_replan_break_even_saturates(oracle_lib):
+    """Section IV-D break-even requests = ceil(cost * epoch / gain), computed
+    here in exact integers; where it does not fit in int64 the oracle reports
+    INT64_MAX (the library's reading), elsewhere the exact value."""
+    rng = np.random.default_rng(91)
+    seen_big = seen_exact = 0
+    for trial in range(12):
+        # unit demand keeps the gain small next to the one-time cost
+        inst = wl.random_small(rng, 30, 3, trial % 2, k_max=8, w_max=1, demand_max=1)
+        prob = _prob(oracle_lib, inst)
+        old = oracle_lib.plan(prob, 1, 0, orders=np.array([[2, 1, 0]], np.int32), threads=1,
+                              safeguards=False).placement
+        epoch = (1 << 63) - 1 if trial % 3 else 30000
+        r = oracle_lib.replan(prob, old, 2, 2, epoch, 1, threads=1)
+        gain = r.new_objective - r.incumbent_objective
+        if gain <= 0:
+            assert r.break_even_requests == -1
+            continue
+        exact = -(-(r.materialization_cost * epoch) // gain)
+        if exact > (1 << 63) - 1:
+            seen_big += 1
+            assert r.break_even_requests == (1 << 63) - 1
+        else:
+            seen_exact += 1
+            assert r.break_even_requests == exact
+    assert seen_big >= 2 and seen_exact >= 2
