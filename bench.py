@@ -2,28 +2,39 @@
 """Planner benchmark: PrefixPlace's coordinate-refined plan on one GB300.
 
 One step = one whole plan (pp_plan_run: standalone-score orders, WorkerGreedy
-pass, up to R refinement sweeps over S starts, objective + argmax) on the
-paper-scale synthetic workload (n = 50,000 chunks, W = 16 workers,
-k = 4,096 slots, 16 starts, 6 rounds), inputs resident in HBM.
+pass, up to R refinement sweeps over S starts, objective + argmax) of the
+headline workload, the paper-scale synthetic instance (n = 50,000 chunks,
+W = 16 workers, k = 4,096 slots, 16 starts, 6 rounds), inputs resident in HBM.
 
   value     Eq. 9 cell updates executed (sum over DPs of n * k_h) per second of
             device time, summed over ranks; L2 is flushed between steps
   e2e       the same metric through the C ABI from pinned host buffers:
             pp_instance_create (upload + tables) + pp_plan_run (placement
             back to the host) + pp_instance_destroy, every step
-  roofline  the tree-DP kernel (dominant), timed live with CUDA events on the
-            launching stream at the plan's launch configuration
-  cpu_baseline  the CPU oracle on a bounded sample of the same workload
+  roofline  the tree-DP step (dominant): the algorithmic bytes of the paper's
+            table algorithm (decision bits n(k+1)/8, p/w/next 16n, every
+            pushed skip row written and read once 16(k+1) per push, the
+            traceback's at most n states 8n) per DP, times the DPs of a step,
+            over the step's CUDA-event time, against the measured HBM copy
+            bandwidth; the dependent row chain that actually limits the kernel
+            is reported beside it (t_row_min)
+  cpu_baseline  the CPU oracle's whole plan of the same workload on the
+            host's cores (one thread per start), outside the timed region
+  configs   the same measurements for all five synthetic workloads (tiny,
+            RAG, source-dependent, paper-scale, stress), each with its oracle
+            baseline (the whole plan, or a bounded sample for the stress one)
 
 --impl reference runs the oracle (the only reference implementation of this
 path) on the host cores and prints the same line with "impl": "reference".
-Multi-GPU (torchrun): weak scaling, 16 starts per GPU out of 16 x N default
-start orders; rank r plans the starts s with s % N == r and the candidates
-are compared once after the timed region (no exchange while planning).
+Multi-GPU (torchrun): --scaling weak (default) plans 16 starts per GPU out of
+16 x N default start orders, --scaling strong splits the 16 starts of one
+plan; rank r plans the starts s with s % N == r and the candidates are
+compared once after the timed region (no exchange while planning).
 """
 from __future__ import annotations
 
 import argparse
+import ctypes
 import hashlib
 import json
 import os
@@ -31,6 +42,7 @@ import statistics
 import subprocess
 import sys
 import tempfile
+import threading
 import time
 
 import numpy as np
@@ -43,10 +55,12 @@ os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
 
 METRIC = "tree-DP cell-updates/s and end-to-end plan time (n=50k, 16 workers) vs HBM roofline"
 UNIT = "cell-updates/s"
-BENCH_CONFIG = 3            # the n = 50,000 / W = 16 / k = 4,096 workload
+HEADLINE_CONFIG = 3         # the n = 50,000 / W = 16 / k = 4,096 workload
 SM_COUNT = 152
 INT32_LANES_PER_SM = 64     # integer add/compare/select/logic: 16 lanes per scheduler, 4 schedulers
 ALU_OPS_PER_CELL = 6        # int64 add, compare, select = 2 + 2 + 2 int32 lane operations
+# side configurations: (warm-up plans, timed plans, timed end-to-end plans)
+SIDE_STEPS = {0: (3, 5, 3), 1: (3, 5, 3), 2: (3, 5, 3), 4: (3, 1, 1)}
 
 
 def _peaks():
@@ -109,34 +123,72 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# --------------------------------------------------------------------------- byte models
+def table_bytes(parent, k: int):
+    """Algorithmic bytes of one Eq. 9 DP of budget k over the whole tree, for
+    the paper's table algorithm (Theorem 1): B_min = decision bits n(k+1)/8 +
+    p, w, next of every row 16n + every skip row that a later row reads,
+    written once and read once, 16(k+1) per push of the tree's stack plan +
+    the traceback's at most n visited states, 8n; B_stream adds the per-row
+    gather of D[next(i)] ((k+1) int64 words) for every internal row
+    (next(i) != i + 1), as a table algorithm that streams rows from memory
+    reads it."""
+    from paper_2608_01655_gb300 import binding as pp
+    order, nxt, skipc, pushl, depth = pp.pp_row_plan(parent)
+    n = len(parent)
+    n_push = int((pushl >= 0).sum())
+    n_internal = int((nxt != np.arange(n) + 1).sum())
+    bmin = n * (k + 1) / 8 + 16 * n + 16 * (k + 1) * n_push + 8 * n
+    bstream = bmin + 8 * (k + 1) * n_internal
+    return {"bmin_bytes_per_dp": bmin, "bstream_bytes_per_dp": bstream, "n_push": n_push,
+            "n_internal": n_internal}
+
+
 # --------------------------------------------------------------------------- oracle legs
-def oracle_sample(inst, starts: int, threads: int):
-    """The oracle as it stands: a greedy pass (no refinement) of `starts`
-    start orders, one thread per start.  Returns (cells, seconds)."""
+def _host_cores():
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+
+
+def oracle_plan(inst, threads: int):
+    """The oracle's whole plan of the workload (default orders, its own
+    standalone-score DPs, safeguards where they apply), one thread per start
+    up to `threads`.  Returns (result, seconds)."""
     import oracle
     prob = oracle.Problem.from_instance(inst)
-    orders = np.stack([np.roll(np.arange(inst.W), s) for s in range(starts)]).astype(np.int32)
     t0 = time.perf_counter()
-    r = oracle.plan(prob, starts, 0, orders=orders, threads=threads)
-    return r.cells, time.perf_counter() - t0
+    r = oracle.plan(prob, inst.starts, inst.rounds, threads=threads)
+    return r, time.perf_counter() - t0
 
 
-def oracle_update(inst, prob, rng):
-    """One oracle worker update (marginals + RootedDP) from a random
-    mid-plan state.  Returns (cells, seconds)."""
+def oracle_updates(inst, count: int, seed: int = 0):
+    """A bounded sample: `count` oracle worker updates (Eq. 7 / Eq. 10
+    marginals + Eq. 9 DP + backtrack), each against its own random holder
+    sets (every worker holds ~5% of the chunks, as in the middle of a plan),
+    run concurrently on `count` threads (the oracle releases the interpreter
+    while it works).  Returns (cells, seconds)."""
     import oracle
-    pl = (rng.random((inst.W, inst.n)) < 0.05).astype(np.uint8)
-    h = int(rng.integers(inst.W))
+    prob = oracle.Problem.from_instance(inst)
+    rng = np.random.default_rng(seed)
+    jobs = []
+    for x in range(count):
+        pl = (rng.random((inst.W, inst.n)) < 0.05).astype(np.uint8)
+        jobs.append((int(rng.integers(inst.W)), pl))
+    cells = sum(inst.n * int(inst.budget[h]) for h, _ in jobs)
+    threads = [threading.Thread(target=oracle.worker_update, args=(prob, h, pl)) for h, pl in jobs]
     t0 = time.perf_counter()
-    oracle.worker_update(prob, h, pl)
-    return inst.n * int(inst.budget[h]), time.perf_counter() - t0
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    return cells, time.perf_counter() - t0
 
 
-def _config(inst, S):
+def _config(inst, S, world=1, scaling="weak"):
     """The workload of both arms (the reference arm times the oracle on it)."""
+    par = (f"starts ({scaling}: {S} per GPU)" if scaling == "weak" else f"starts ({scaling}: {S} over {world} GPUs)")
     return {"workload": inst.name, "n": inst.n, "W": inst.W, "k": int(inst.budget.max()), "starts": S,
             "rounds": inst.rounds, "mode": "source-dependent" if inst.mode else "requester-side",
-            "l2": "flushed between steps (256 MiB write)", "parallelism": f"starts (weak, {S} per GPU)"}
+            "l2": "flushed between steps (256 MiB write)", "parallelism": par}
 
 
 def run_reference(args):
@@ -146,27 +198,26 @@ def run_reference(args):
     from paper_2608_01655_gb300 import workloads as wl
     import oracle
     oracle.build()
-    inst = wl.make(BENCH_CONFIG)
-    prob = oracle.Problem.from_instance(inst)
-    rng = np.random.default_rng(0)
-    for _ in range(args.warmup):
-        oracle_update(inst, prob, rng)
+    inst = wl.make(args.config)
+    cores = _host_cores()
+    oracle_updates(inst, cores, seed=10_000)           # warm the page cache and the library
+    for w in range(args.warmup):
+        oracle_updates(inst, cores, seed=w)
     cells = 0
     secs = 0.0
-    times = []
-    for _ in range(args.steps):
-        c, s = oracle_update(inst, prob, rng)
+    for s in range(args.steps):
+        c, t = oracle_updates(inst, cores, seed=1000 + s)
         cells += c
-        secs += s
-        times.append(s)
+        secs += t
     value = cells / secs
-    sample = f"one worker update (Eq. 7 marginals + Eq. 9 DP + backtrack, {inst.n} x {int(inst.budget[0])} cells) per step"
+    sample = (f"{cores} oracle worker updates per step, one per host core, concurrently "
+              f"(Eq. 7/10 marginals + Eq. 9 DP + backtrack, {inst.n} x {int(inst.budget[0])} cells each)")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * secs / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
-        "data": "synthetic", "config": _config(inst, inst.starts),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "higher_is_better": True, "scaling": args.scaling, "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic", "config": _config(inst, inst.starts, args.gpus, args.scaling),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "gpu_launches": 0,
     }
@@ -182,7 +233,7 @@ def _dist():
     return world, rank, local
 
 
-TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "tree_dp_traffic_paper-n50000-W16-k4096.md")
+TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "k_tree_dp_wave_traffic_paper-n50000-k4096.md")
 DP_SOURCES = [os.path.join(ROOT, "paper_2608_01655_gb300", "csrc", f) for f in ("pp_dp.cu", "pp_internal.cuh")]
 
 
@@ -194,9 +245,9 @@ def dp_source_sha256():
 
 
 def _traffic_record():
-    """Per-launch DRAM traffic of the tree-DP launch from the committed ncu
-    summary (its `traffic_record:` line), used only while the DP sources are
-    unchanged since the counters were taken."""
+    """DRAM traffic per swept cell of the tree-DP kernel from the committed
+    one-kernel ncu capture (its `traffic_record:` line), used only while the DP
+    sources are unchanged since the counters were taken."""
     try:
         for line in open(TRAFFIC_SUMMARY):
             if line.startswith("traffic_record:"):
@@ -207,29 +258,38 @@ def _traffic_record():
     return None
 
 
-def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, stream):
-    """Read bandwidth of L2 and HBM (pp_probe_read), the per-row time of the
-    smallest DP launch shape (one warp per DP, 32 columns: the dependent row
-    chain with no hand-off between warps), and the B_stream model of the
-    paper's table algorithm (every row with next(i) != i+1 gathers a whole
-    skip row from memory)."""
+def _probe_read_gbs(torch, stream, nbytes, iters):
+    """Read bandwidth of a device buffer (libpp_probe.so, the benchmark's
+    bandwidth probe; not part of the planner)."""
+    from paper_2608_01655_gb300 import build
+    lib = ctypes.CDLL(build.PROBE_LIB)
+    lib.pp_probe_read.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int32, ctypes.c_void_p,
+                                  ctypes.c_void_p]
+    lib.pp_probe_read.restype = ctypes.c_int
     sink = torch.zeros(1, dtype=torch.int64, device="cuda")
+    buf = torch.ones(nbytes // 8, dtype=torch.int64, device="cuda")
+    sp = ctypes.c_void_p(stream.cuda_stream)
 
-    def read_gbs(nbytes, iters):
-        buf = torch.ones(nbytes // 8, dtype=torch.int64, device="cuda")
-        pp.pp_probe_read(buf, 1, sink, stream)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        pp.pp_probe_read(buf, iters, sink, stream)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        del buf
-        return nbytes * iters / (e0.elapsed_time(e1) / 1000.0) / 1e9
+    def call(it):
+        rc = lib.pp_probe_read(ctypes.c_void_p(buf.data_ptr()), nbytes, it, ctypes.c_void_p(sink.data_ptr()), sp)
+        if rc != 0:
+            raise RuntimeError(f"pp_probe_read failed ({rc})")
 
-    l2_gbs = read_gbs(32 << 20, 200)          # 32 MiB: resident in L2
-    hbm_gbs = read_gbs(4 << 30, 3)            # 4 GiB: far larger than L2
+    call(1)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    call(iters)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    del buf
+    return nbytes * iters / (e0.elapsed_time(e1) / 1000.0) / 1e9
 
-    # t_row_min: the plan's last DP inputs at one warp per DP and 32 columns
+
+def _t_row_min(pp, torch, inst, ppi, res, S, stream):
+    """Per-row time of the smallest DP launch shape (one warp per DP, 32
+    columns, no hand-off between warps) on the plan's last marginals: the
+    dependent row chain alone."""
+    n = inst.n
     masks = np.zeros((S, n), np.uint32)
     for m in range(inst.W):
         masks |= res.placement[m].astype(np.uint32) << np.uint32(m)
@@ -238,7 +298,7 @@ def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, s
     prof = torch.zeros((S, n), dtype=torch.int64, device="cuda")
     pp.pp_marginals(ppi, workers, masks_t, prof)
     kk = 32
-    pp.pp_tune_dp(1, 1, False, False)
+    pp.pp_tune_dp(ppi, 1, 1, False, False)
     try:
         bud = torch.full((S,), kk, dtype=torch.int32, device="cuda")
         best = torch.zeros(S, dtype=torch.int64, device="cuda")
@@ -255,25 +315,99 @@ def _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, s
         ppi.sync()
         rows_max = int(pp.pp_dp_rows_swept(ppi, S, kk, bits).max())
     finally:
-        pp.pp_tune_dp(0, 0, False, False)
-    t_row_min = min(ts) / rows_max
-    # B_stream: B_min plus one (k+1)-word skip-row read for every row whose
-    # skip row is not the row just computed
-    code = pp.pp_row_plan_registers(inst.parent, inst.weight)
-    frac_gather = float(np.mean(((code >> 3) & 3) != 0))
-    bstream = bmin + rows_swept * frac_gather * 8 * (k + 1)
-    rows_item = rows_swept / items
-    return {
-        "l2_read_gbs": l2_gbs, "hbm_read_gbs": hbm_gbs,
-        "roofline_extra": {
-            "bstream_bytes_per_launch": bstream, "bstream_gbs": bstream / dp_t / 1e9,
-            "bstream_frac_of_l2": bstream / dp_t / 1e9 / l2_gbs,
-            "l2_read_gbs_probe": l2_gbs, "hbm_read_gbs_probe": hbm_gbs,
-            "t_row_min_ns": 1e9 * t_row_min,
-            "t_row_min_source": "one warp per DP, 32 columns, same rows (pp_tune_dp(1, 1))",
-            "t_dp_over_rows_x_t_row_min": dp_t / (rows_item * t_row_min),
-        },
+        pp.pp_tune_dp(ppi, 0, 0, False, False)
+    return min(ts) / rows_max
+
+
+def measure_plan(pp, torch, ppi, S, R, orders, warmup, steps, flush, stream, sched, sg, barrier=None):
+    """`warmup` untimed plans, then `steps` plans timed with CUDA events on
+    the launching stream, L2 flushed before each.  Returns (last result,
+    per-step seconds, summed phase ms)."""
+    res = None
+    for _ in range(warmup):
+        res = pp.pp_plan_run(ppi, S, orders, R, safeguards=sg, schedule=sched)
+    times, phase = [], [0.0, 0.0, 0.0]
+    for _ in range(steps):
+        flush.fill_(1)
+        if barrier:
+            barrier()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        # events around every launch of the plan (read after the plan returns);
+        # the NVTX range lets a profiler select the timed plans' launches
+        torch.cuda.nvtx.range_push("timed_plan")
+        res = pp.pp_plan_run(ppi, S, orders, R, time_phases=True, safeguards=sg, schedule=sched)
+        torch.cuda.nvtx.range_pop()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if barrier:
+            barrier()
+        times.append(e0.elapsed_time(e1) / 1000.0)
+        for x in range(3):
+            phase[x] += res.phase_ms[x]
+    return res, times, phase
+
+
+def measure_e2e(pp, torch, inst, S, R, orders, warmup, steps, flush, sched, sg, objective):
+    """The plan through the C ABI from pinned host buffers, every step:
+    instance creation (upload + tables), pp_plan_run (placement back to the
+    host), instance destruction.  Returns (per-step seconds, h2d bytes,
+    d2h bytes)."""
+    host = {}
+    for name in ("parent", "weight", "demand", "recompute", "transfer", "budget"):
+        a = np.ascontiguousarray(getattr(inst, name))
+        host[name] = torch.from_numpy(a).pin_memory().numpy()
+    h2d = sum(v.nbytes for v in host.values())
+    d2h = inst.W * inst.n + 8 * (S * 3 + 1)
+    times = []
+    for it in range(warmup + steps):
+        flush.fill_(3)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        with pp.Instance(host["parent"], host["weight"], host["demand"], host["recompute"],
+                         host["transfer"], inst.mode, host["budget"]) as ppe:
+            r2 = pp.pp_plan_run(ppe, S, orders, R, safeguards=sg, schedule=sched)
+        torch.cuda.synchronize()
+        if it >= warmup:
+            times.append(time.perf_counter() - t0)
+        assert r2.objective == objective
+    return times, h2d, d2h
+
+
+def plan_summary(inst, res, times, phase, e2e_times, h2d, d2h, l2_gbs, hbm_gbs):
+    """Per-workload figures: plan time with inputs resident and with upload,
+    executed and swept cells/s, per-update latency, and the table
+    algorithm's B_min / B_stream bytes over the DP step's time as fractions
+    of the HBM copy and L2 read bandwidths."""
+    k = int(inst.budget.max())
+    plan_s = sum(times) / len(times)
+    nl = max(res.dp_launches, 1)
+    dp_t = phase[1] / 1000.0 / (nl * len(times))
+    items = res.dp_count / nl
+    tb = table_bytes(inst.parent, k)
+    out = {
+        "workload": inst.name, "n": inst.n, "W": inst.W, "k": k, "starts": inst.starts, "rounds": inst.rounds,
+        "mode": "source-dependent" if inst.mode else "requester-side",
+        "steps": len(times), "plan_ms": 1000 * plan_s,
+        "plan_ms_with_upload": 1000 * sum(e2e_times) / len(e2e_times) if e2e_times else None,
+        "e2e_steps": len(e2e_times), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+        "cells_per_s_executed": res.dp_cells / plan_s,
+        "cells_per_s_swept": res.dp_rows_swept * k / plan_s,
+        "update_ms": sum(phase) / (nl * len(times)),
+        "dp_step_ms": 1000 * dp_t, "dps_per_step": items,
+        "phase_ms": {"marginals": phase[0] / len(times), "tree_dp": phase[1] / len(times),
+                     "traceback_accept": phase[2] / len(times)},
+        **tb,
+        "bmin_gbs": items * tb["bmin_bytes_per_dp"] / dp_t / 1e9,
+        "bmin_frac_of_hbm": items * tb["bmin_bytes_per_dp"] / dp_t / 1e9 / hbm_gbs,
+        "bstream_frac_of_l2": items * tb["bstream_bytes_per_dp"] / dp_t / 1e9 / l2_gbs,
+        "objective": res.objective, "best_start": res.best_start,
+        "sweeps": res.per_start_sweeps.tolist(), "dp_count": res.dp_count, "dp_cells": res.dp_cells,
+        "dp_rows_swept": res.dp_rows_swept, "schedule": "per-start streams" if res.schedule == 2 else "lock step",
     }
+    return out
 
 
 def _extras(pp, torch, wl, inst, res):
@@ -325,6 +459,46 @@ def _extras(pp, torch, wl, inst, res):
     return out
 
 
+def side_config(pp, torch, wl, cfg, flush, stream, sched, l2_gbs, hbm_gbs, with_oracle):
+    """Plan, end-to-end and oracle figures of one more workload (single GPU)."""
+    inst = wl.make(cfg)
+    warm, steps, e2e_steps = SIDE_STEPS[cfg]
+    sg = True
+    with pp.Instance.from_workload(inst) as ppi:
+        res, times, phase = measure_plan(pp, torch, ppi, inst.starts, inst.rounds, None, warm, steps, flush,
+                                         stream, sched, sg)
+    e2e_times, h2d, d2h = measure_e2e(pp, torch, inst, inst.starts, inst.rounds, None, 0, e2e_steps, flush,
+                                      sched, sg, res.objective)
+    out = plan_summary(inst, res, times, phase, e2e_times, h2d, d2h, l2_gbs, hbm_gbs)
+    out["warmup"] = warm
+    if with_oracle:
+        out["oracle"] = oracle_leg(inst, res)
+    return out
+
+
+def oracle_leg(inst, res):
+    """The oracle on the host cores: the whole plan where it finishes in
+    seconds (cross-checked against the GPU plan's objective and placement), a
+    bounded sample of concurrent worker updates for the stress workload."""
+    cores = _host_cores()
+    if inst.n * int(inst.budget.max()) * inst.W * inst.starts * (1 + inst.rounds) > 2e12:
+        count = min(cores, 16)
+        cells, secs = oracle_updates(inst, count, seed=7)
+        rate = cells / secs
+        return {"kind": "oracle sample", "cores": count, "value": rate, "unit": UNIT,
+                "sample": f"{count} concurrent worker updates (marginals + Eq. 9 DP + backtrack, "
+                          f"{inst.n} x {int(inst.budget.max())} cells each), {secs:.1f} s",
+                "plan_s_extrapolated": res.dp_cells / rate,
+                "extrapolation": "the GPU plan's executed cells at the sample's rate"}
+    threads = min(inst.starts, cores)
+    r, secs = oracle_plan(inst, threads)
+    return {"kind": "oracle plan", "cores": threads, "value": r.cells / secs, "unit": UNIT, "plan_s": secs,
+            "cells": r.cells, "sample": f"the whole plan ({inst.starts} starts, {inst.rounds} rounds), "
+                                        f"one thread per start",
+            "objective_equal": r.objective == res.objective, "best_start_equal": r.best_start == res.best_start,
+            "placement_equal": bool(np.array_equal(r.placement, res.placement))}
+
+
 def run_native(args):
     import torch
     world, rank, local = _dist()
@@ -335,19 +509,19 @@ def run_native(args):
     else:
         torch.cuda.set_device(0)
     from paper_2608_01655_gb300 import binding as pp
+    from paper_2608_01655_gb300 import shard
     from paper_2608_01655_gb300 import workloads as wl
 
-    inst = wl.make(BENCH_CONFIG)
+    inst = wl.make(args.config)
     S, R = inst.starts, inst.rounds
     stream = torch.cuda.current_stream()
     ppi = pp.Instance.from_workload(inst)
-    orders = None
+    orders, my_idx = None, np.arange(S)
     if world > 1:
-        # weak scaling: S starts per GPU out of S * world default orders, the
-        # same on every rank; rank r plans the starts s with s % world == r
-        from paper_2608_01655_gb300 import shard
-        all_orders = pp.pp_default_orders(ppi, S * world)
-        orders = all_orders[shard.my_starts(S * world, rank, world)]
+        # every rank computes the same default orders; rank r plans s % world == r
+        orders, my_idx = shard.rank_orders(lambda total: pp.pp_default_orders(ppi, total), S, rank, world,
+                                           args.scaling)
+    S_mine = len(my_idx) if world > 1 else S
     # the requester-side safeguards are candidates of the whole plan, not of a
     # start: with several ranks only the starts are sharded and compared
     sg = world == 1
@@ -358,156 +532,153 @@ def run_native(args):
             torch.distributed.barrier()
 
     sched = {"auto": 0, "lock": 1, "per-start": 2}[args.schedule]
-    res = None
-    for _ in range(args.warmup):
-        res = pp.pp_plan_run(ppi, S, orders, R, safeguards=sg, schedule=sched)
-    cells_per_plan = res.dp_cells
-    launches_per_plan = res.kernel_launches
-    times, phase_sum = [], [0.0, 0.0, 0.0]
     with ClockSampler(local) as clk:
-        for _ in range(args.steps):
-            flush.fill_(1)
-            barrier()
-            torch.cuda.synchronize()
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            # events around every launch of the plan (read after the plan returns);
-            # the NVTX range lets a profiler select the timed plans' launches
-            torch.cuda.nvtx.range_push("timed_plan")
-            res = pp.pp_plan_run(ppi, S, orders, R, time_phases=True, safeguards=sg, schedule=sched)
-            torch.cuda.nvtx.range_pop()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            barrier()
-            times.append(e0.elapsed_time(e1) / 1000.0)
-            for x in range(3):
-                phase_sum[x] += res.phase_ms[x]
+        res, times, phase = measure_plan(pp, torch, ppi, S_mine, R, orders, args.warmup, args.steps, flush, stream,
+                                         sched, sg, barrier=barrier)
     clocks = clk.summary()
     total = sum(times)
+    cells_mine = res.dp_cells * args.steps
     if world > 1:
-        t = torch.tensor([total], dtype=torch.float64, device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total = float(t.item())
-    value = world * cells_per_plan * args.steps / total
+        t = torch.tensor([total, float(cells_mine)], dtype=torch.float64, device="cuda")
+        tm = t.clone()
+        torch.distributed.all_reduce(tm, op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.SUM)
+        total, cells_all = float(tm[0].item()), float(t[1].item())
+    else:
+        cells_all = float(cells_mine)
+    value = cells_all / total
 
-    # ---- the dominant kernel: the plan's batched tree-DP launches (row pruning
-    # + Eq. 9 sweep), CUDA events on the launching stream over the timed region
-    k = int(inst.budget.max())
-    n = inst.n
-    nl = res.dp_launches
-    dp_t = phase_sum[1] / 1000.0 / (nl * args.steps)              # s per launch
-    items = res.dp_count / nl                                      # DPs per launch
-    cells_launch = res.dp_cells / nl                               # n x k table cells per launch
-    rows_swept = res.dp_rows_swept / nl                            # kept rows per launch
-    cells_swept = rows_swept * k
+    # ---- the dominant kernel: the plan's tree-DP steps (row pruning + Eq. 9
+    # sweep), CUDA events on the launching streams over the timed region
     peaks, peak_kind = _peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    k = int(inst.budget.max())
+    nl = max(res.dp_launches, 1)
+    dp_t = phase[1] / 1000.0 / (nl * args.steps)               # s per DP step
+    items = res.dp_count / nl                                   # DPs per step
+    rows_swept = res.dp_rows_swept / nl
+    cells_swept = rows_swept * k
+    tb = table_bytes(inst.parent, k)
+    bmin_step = items * tb["bmin_bytes_per_dp"]
+    achieved = bmin_step / dp_t / 1e9
+    l2_gbs = _probe_read_gbs(torch, stream, 32 << 20, 200)     # 32 MiB: resident in L2
+    hbm_read_gbs = _probe_read_gbs(torch, stream, 4 << 30, 3)  # 4 GiB: far larger than L2
+    t_row_min = _t_row_min(pp, torch, inst, ppi, res, S_mine, stream)
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = SM_COUNT * INT32_LANES_PER_SM * sm_mhz * 1e6 / ALU_OPS_PER_CELL   # cells/s
-    achieved = cells_swept / dp_t                 # cells the kernel actually computed
-    # algorithmic bytes of one launch: decision bits of the swept rows + p/w/next
-    # of every row + skip-row pushes
-    order, nxt, skipc, pushl, depth = pp.pp_row_plan(inst.parent)
-    pushes = int((pushl >= 0).sum())
-    bmin = rows_swept * (k + 1) / 8 + items * (16 * n + 16 * (k + 1) * pushes)
     tr = _traffic_record()
     traffic = None
-    if tr and tr.get("cells_swept_per_launch"):
-        traffic = tr["bytes_per_launch"] * cells_swept / tr["cells_swept_per_launch"]
+    if tr and tr.get("bytes_per_swept_cell"):
+        traffic = tr["bytes_per_swept_cell"] * cells_swept
     per_start = res.schedule == 2
-    roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": alu_peak / 1e12, "unit": "Tcell/s",
-                "frac": achieved / alu_peak, "traffic": traffic,
-                "peak_source": f"derived: {SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 ALU lanes x "
-                               f"{sm_mhz:.0f} MHz / {ALU_OPS_PER_CELL} int32 ops per cell ({peak_kind} clock)",
-                "kernel": ("k_prune + k_tree_dp_wave (one tree-DP step of the plan: every start's DP on its "
-                           "own stream, concurrently; duration = mean over starts of the start's DP events)"
-                           if per_start else "k_prune + k_tree_dp_wave (one batched tree-DP launch of the plan)"),
-                "launches": nl * args.steps, "launch_ms": 1000 * dp_t, "items_per_launch": items,
-                "cells_per_launch": cells_launch, "cells_swept_per_launch": cells_swept,
-                "rows_swept_per_launch": rows_swept,
-                "hbm_bmin_gbs": bmin / dp_t / 1e9,
-                "hbm_bmin_frac": bmin / dp_t / 1e9 / float(peaks.get("hbm_gbs", 6800.0)),
-                "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0)), "hbm_peak_kind": peak_kind}
-
-    # ---- memory-hierarchy probes and the dependent-row bound (outside the timed region)
-    probes = _probes(pp, torch, inst, ppi, res, S, k, n, dp_t, rows_swept, items, bmin, stream)
-    roofline.update(probes.pop("roofline_extra"))
+    roofline = {
+        "bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+        "traffic": traffic,
+        "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind} copy bandwidth)",
+        "achieved_source": ("algorithmic bytes of the paper's table algorithm per DP (bmin_bytes_per_dp: "
+                            "n(k+1)/8 decision bits + 16n p/w/next + 16(k+1) per skip-row push + 8n "
+                            "traceback) x DPs per step / the step's CUDA-event time"),
+        "traffic_source": ("DRAM bytes per swept cell of a one-kernel ncu capture of the batched DP on the "
+                           "small profile case, times the step's swept cells" if traffic is not None else
+                           "no capture of the current DP sources"),
+        "limiter": ("latency: the dependent row chain of Eq. 9 (one warp's rows follow one another; "
+                    "t_dp_over_rows_x_t_row_min compares the step with that chain alone)"),
+        "kernel": ("k_prune + k_tree_dp_wave (one tree-DP step of the plan: every start's DP on its own "
+                   "stream, concurrently; duration = mean over starts of the start's DP events)"
+                   if per_start else "k_prune + k_tree_dp_wave (one batched tree-DP launch of the plan)"),
+        "launches": nl * args.steps, "launch_ms": 1000 * dp_t, "items_per_launch": items,
+        **tb,
+        "bmin_bytes_per_launch": bmin_step,
+        "cells_per_launch": res.dp_cells / nl, "cells_swept_per_launch": cells_swept,
+        "rows_swept_per_launch": rows_swept,
+        "bstream_gbs": items * tb["bstream_bytes_per_dp"] / dp_t / 1e9,
+        "bstream_frac_of_l2": items * tb["bstream_bytes_per_dp"] / dp_t / 1e9 / l2_gbs,
+        "l2_read_gbs_probe": l2_gbs, "hbm_read_gbs_probe": hbm_read_gbs,
+        "t_row_min_ns": 1e9 * t_row_min,
+        "t_row_min_source": "one warp per DP, 32 columns, the same rows (pp_tune_dp(inst, 1, 1))",
+        "t_dp_over_rows_x_t_row_min": dp_t / ((rows_swept / items) * t_row_min),
+        "alu_model": {"achieved_tcells": cells_swept / dp_t / 1e12, "peak_tcells": alu_peak / 1e12,
+                      "frac": cells_swept / dp_t / alu_peak,
+                      "source": (f"derived, not measured: {SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 ALU lanes x "
+                                 f"{sm_mhz:.0f} MHz / {ALU_OPS_PER_CELL} int32 ops per cell; counts only the "
+                                 f"16-lane ALU pipe of each scheduler (adds that issue on the FMA pipe are not "
+                                 f"credited), and only the cells the pruned sweep computes")},
+    }
 
     # ---- end to end through the C ABI from pinned host buffers -------------
-    host = {}
-    for name in ("parent", "weight", "demand", "recompute", "transfer", "budget"):
-        a = np.ascontiguousarray(getattr(inst, name))
-        t = torch.from_numpy(a).pin_memory()
-        host[name] = t.numpy()
-    h2d = sum(v.nbytes for v in host.values())
-    d2h = 4 * n + 8 * (S * 3 + 1)
-    e2e_times = []
-    for it in range(args.warmup + args.steps):
-        flush.fill_(3)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        with pp.Instance(host["parent"], host["weight"], host["demand"], host["recompute"],
-                         host["transfer"], inst.mode, host["budget"]) as ppe:
-            r2 = pp.pp_plan_run(ppe, S, orders, R, safeguards=sg, schedule=sched)
-        torch.cuda.synchronize()
-        if it >= args.warmup:
-            e2e_times.append(time.perf_counter() - t0)
-        assert r2.objective == res.objective
+    e2e_times, h2d, d2h = measure_e2e(pp, torch, inst, S_mine, R, orders, args.warmup, args.steps, flush, sched,
+                                      sg, res.objective)
     e2e_total = sum(e2e_times)
     if world > 1:
         t = torch.tensor([e2e_total], dtype=torch.float64, device="cuda")
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         e2e_total = float(t.item())
-    e2e_value = world * cells_per_plan * args.steps / e2e_total
-
-    extras = _extras(pp, torch, wl, inst, res) if rank == 0 else None
+    e2e_value = cells_all / e2e_total
+    headline = plan_summary(inst, res, times, phase, e2e_times, h2d, d2h, l2_gbs, hbm_peak)
 
     # ---- candidates of all ranks compared once (outside the timed region) ---
     best_obj, best_start = res.objective, res.best_start
     if world > 1:
-        mine = shard.my_starts(S * world, rank, world)
-        won = shard.exchange(res.objective, int(mine[res.best_start]), res.placement)
+        won = shard.exchange(res.objective, int(my_idx[res.best_start]), res.placement)
         best_obj, best_start = won.objective, won.best_start
 
+    extras = _extras(pp, torch, wl, inst, res) if rank == 0 and world == 1 and not args.headline_only else None
+    geometry = {**pp.pp_dp_geometry(ppi, S_mine, k), "split": pp.pp_dp_split(ppi, S_mine, k)}
+    ppi.close()
+
+    # ---- the other four workloads (single GPU) -----------------------------
+    configs = {}
+    if world == 1 and not args.headline_only:
+        for cfg in (0, 1, 2, 4):
+            if cfg != args.config:
+                configs[wl.make(cfg).name] = side_config(pp, torch, wl, cfg, flush, stream, sched, l2_gbs,
+                                                         hbm_peak, not args.no_cpu_baseline)
+
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
-        threads = 2
-        c, s = oracle_sample(inst, threads, threads)
-        cpu = {"value": c / s, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"greedy pass (no refinement) of {threads} start orders, one thread each, "
-                         f"{c} Eq. 9 cells in {s:.1f} s", "host_cores": os.cpu_count()}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        leg = oracle_leg(inst, res)
+        headline["oracle"] = leg
+        cpu = {"value": leg["value"], "unit": UNIT, "cores": leg["cores"], "kind": leg["kind"],
+               "sample": leg["sample"], "host_cores": _host_cores()}
+        for key in ("plan_s", "objective_equal", "best_start_equal", "placement_equal", "plan_s_extrapolated"):
+            if key in leg:
+                cpu[key] = leg[key]
+        cpu["gpu_plan_s"] = sum(times) / len(times)
+    configs = {inst.name: headline, **configs}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": _config(inst, S),
+            "scaling": args.scaling, "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": _config(inst, S, world, args.scaling),
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": 1000 * e2e_total / args.steps},
-            "gpu_launches": launches_per_plan * args.steps,
+            "gpu_launches": res.kernel_launches * args.steps,
             "clocks": clocks,
             "plan": {"objective": best_obj, "best_start": best_start,
                      "schedule": "per-start streams" if per_start else "lock step",
-                     "dp_count": res.dp_count, "dp_cells": cells_per_plan,
+                     "hw_queues_assumed": res.hw_queues,
+                     "dp_count": res.dp_count, "dp_cells": res.dp_cells,
                      "dp_launches": nl, "dp_rows_swept": res.dp_rows_swept,
                      "dp_cells_swept": res.dp_rows_swept * k,
+                     "cells_per_s_swept_here": res.dp_rows_swept * k * args.steps / total,
+                     "starts_planned_here": int(S_mine),
                      "sweeps": res.per_start_sweeps.tolist(),
                      "step_ms": [round(1000 * t, 3) for t in times]},
-            "phase_ms": {"marginals": phase_sum[0] / args.steps, "tree_dp": phase_sum[1] / args.steps,
-                         "traceback_accept": phase_sum[2] / args.steps},
-            "update_ms": sum(phase_sum) / (nl * args.steps),
+            "phase_ms": {"marginals": phase[0] / args.steps, "tree_dp": phase[1] / args.steps,
+                         "traceback_accept": phase[2] / args.steps},
+            "update_ms": sum(phase) / (nl * args.steps),
             "update_note": ("one worker update (marginals + tree DP + traceback/accept) of every start, "
                             "the starts on their own streams (phase times: mean over starts)" if per_start else
                             "one batched worker update (marginals + tree DP + traceback/accept) of all starts"),
-            "probes": probes,
+            "configs": configs,
             "next_steps": extras,
-            "dp_geometry": {**pp.pp_dp_geometry(ppi, S, k), "split": pp.pp_dp_split(ppi, S, k)},
+            "dp_geometry": geometry,
         }
         print(json.dumps(line), flush=True)
-    ppi.close()
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
@@ -515,13 +686,13 @@ def run_native(args):
 
 def run_profile_dp(args):
     """A small case for ncu: marginals, the tree DP and the traceback of
-    `--profile-dp B` items of the paper-scale workload, launched twice (ncu
+    `--profile-dp B` items of the headline workload, launched twice (ncu
     captures the second)."""
     import torch
     torch.cuda.set_device(0)
     from paper_2608_01655_gb300 import binding as pp
     from paper_2608_01655_gb300 import workloads as wl
-    inst = wl.make(BENCH_CONFIG)
+    inst = wl.make(args.config)
     ppi = pp.Instance.from_workload(inst)
     B, n, k = args.profile_dp, inst.n, int(inst.budget.max())
     workers = torch.arange(B, dtype=torch.int32, device="cuda") % inst.W
@@ -536,8 +707,11 @@ def run_profile_dp(args):
         pp.pp_tree_dp(ppi, prof, bud, k, best, bits)
         pp.pp_traceback(ppi, bits, bud, k, chosen)
     ppi.sync()
+    rows = pp.pp_dp_rows_swept(ppi, B, k, bits)
     print(json.dumps({"profile_dp": B, "geometry": pp.pp_dp_geometry(ppi, B, k), "split": pp.pp_dp_split(ppi, B, k),
-                      "best": best.tolist()}))
+                      "rows_swept": rows.tolist(), "cells_swept": int(rows.sum()) * k,
+                      "dp_src_sha256": dp_source_sha256(), "best": best.tolist()}))
+    ppi.close()
     return 0
 
 
@@ -547,6 +721,12 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--config", type=int, default=HEADLINE_CONFIG, choices=range(5),
+                    help="headline workload (0 tiny, 1 RAG, 2 source-dependent, 3 paper-scale, 4 stress)")
+    ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
+                    help="with several GPUs: weak = 16 starts per GPU, strong = the 16 starts of one plan split")
+    ap.add_argument("--headline-only", action="store_true",
+                    help="skip the other four workloads and the side timings")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=["auto", "lock", "per-start"], default="auto",
                     help="plan schedule: automatic (per-start streams when the hardware queues allow), "

@@ -92,6 +92,12 @@ typedef struct {
                                       when the CUDA context is created) gives every stream its
                                       own hardware queue, min(S, 32), else lock step.
                                       out: the schedule used (1 or 2).  Results are identical */
+    int32_t hw_queues;             /* out: the hardware queue count the automatic schedule assumed
+                                      (CUDA_DEVICE_MAX_CONNECTIONS as read at the call, 8 when
+                                      unset).  The driver reads that variable only when the CUDA
+                                      context is created, so a context created before it was set
+                                      may have fewer queues: the per-start schedule then runs
+                                      slower, with the same results */
 } pp_plan_stats;
 
 /*
@@ -348,15 +354,26 @@ pp_status pp_dp_geometry(const pp_instance *inst, int32_t batch, int32_t max_bud
 pp_status pp_dp_split(const pp_instance *inst, int32_t batch, int32_t max_budget, int32_t *out);
 
 /*
- * pp_tune_dp -- process-wide override of the DP launch shape, for tuning
- * sweeps: CTAs per cluster (1..8, 0 = automatic), columns per thread (power
- * of two up to 16, 0 = automatic), force_flat != 0 selects the one-CTA kernel,
- * no_prune != 0 sweeps every row instead of the pruned sweep (results are the
- * same either way).  Later pp_dp_bits_size / pp_tree_dp / pp_traceback /
- * pp_plan_run calls use it, so set it before sizing workspaces.
- * Errors: PP_EINVAL.
+ * pp_dp_stack_bytes -- bytes of skip-row stack scratch the instance holds
+ * (no counterpart in the paper; host out).  pp_tree_dp and pp_plan_run
+ * allocate it on the first launch whose skip-row stack does not fit in shared
+ * memory and keep it until pp_instance_destroy; pp_tree_dp_noalloc never adds
+ * to it.  0 before any such launch.  Errors: PP_EINVAL.
  */
-pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
+pp_status pp_dp_stack_bytes(const pp_instance *inst, size_t *out);
+
+/*
+ * pp_tune_dp -- override of this instance's DP launch shape, for tuning
+ * sweeps (no counterpart in the paper): CTAs per cluster (1..8, 0 =
+ * automatic), columns per thread (power of two up to 16, 0 = automatic),
+ * force_flat != 0 selects the one-CTA kernel, no_prune != 0 sweeps every row
+ * instead of the pruned sweep (results are the same either way).  Later
+ * pp_dp_bits_size / pp_tree_dp / pp_traceback / pp_plan_run calls on this
+ * instance use it, so set it before sizing workspaces; other instances are
+ * not affected.  Not thread-safe against concurrent calls on the same
+ * instance.  Errors: PP_EINVAL.
+ */
+pp_status pp_tune_dp(pp_instance *inst, int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
                      int32_t no_prune);
 
 /*
@@ -369,17 +386,6 @@ pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t f
  * Synchronous.  Errors: PP_EINVAL, PP_ENOMEM, PP_ECUDA.
  */
 pp_status pp_default_orders(pp_instance *inst, int32_t n_starts, int32_t *orders, void *stream);
-
-/*
- * pp_probe_read -- benchmark helper with no counterpart in the paper: reads
- * the device buffer `buf` (`bytes` bytes, 16-byte aligned, a multiple of 16)
- * `iters` times with 16-byte loads that bypass L1, on all SMs.  A buffer that
- * fits in L2 gives the L2 read bandwidth that the roofline of the DP's
- * skip-row gathers is quoted against; a buffer far larger than L2 gives the
- * HBM read bandwidth.  `sink` (device, 8 bytes) only keeps the loads live.
- * Asynchronous on `stream`.  Errors: PP_EINVAL, PP_ECUDA.
- */
-pp_status pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *sink, void *stream);
 
 /*
  * pp_safeguards -- the safeguard candidates that Algorithm 1 adds for the

@@ -53,7 +53,7 @@ class PlanStats(ctypes.Structure):
                 ("kernel_launches", _i32), ("dp_rows_swept", _i64), ("time_phases", _i32),
                 ("phase_ms", ctypes.c_float * 3), ("dp_launches", _i32), ("no_safeguards", _i32),
                 ("safeguard_objective", ctypes.c_int64 * 3), ("marginals", _i32), ("used_top2", _i32),
-                ("schedule", _i32)]
+                ("schedule", _i32), ("hw_queues", _i32)]
 
 
 _SIGS = {
@@ -71,11 +71,11 @@ _SIGS = {
     "pp_test_inject": [_i32, _i32],
     "pp_dp_geometry": [_P, _i32, _i32, _P],
     "pp_dp_split": [_P, _i32, _i32, _P],
-    "pp_tune_dp": [_i32, _i32, _i32, _i32],
+    "pp_tune_dp": [_P, _i32, _i32, _i32, _i32],
     "pp_tree_dp_noalloc": [_P, _i32, _P, _P, _i32, _P, _P, _P],
     "pp_dp_rows_swept": [_P, _i32, _i32, _P, _P, _P],
+    "pp_dp_stack_bytes": [_P, ctypes.POINTER(ctypes.c_size_t)],
     "pp_default_orders": [_P, _i32, _P, _P],
-    "pp_probe_read": [_P, ctypes.c_size_t, _i32, _P, _P],
     "pp_safeguards": [_P, _P, _P, _P],
     "pp_replan": [_P, _P, _i32, _P, _i32, _i64, _i64, _P, _P, _P, _P],
 }
@@ -254,6 +254,7 @@ class PlanResult:
     safeguard_objective: tuple = ()     # Independent, Popularity, LocalDedup (requester-side)
     used_top2: bool = False             # source-dependent marginals from top-2 holder tables
     schedule: int = 0                   # 1 lock step, 2 per-start streams
+    hw_queues: int = 0                  # hardware queues the automatic schedule assumed
 
 
 def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0, stream=None,
@@ -287,7 +288,7 @@ def pp_plan_run(inst: Instance, n_starts: int, orders=None, max_rounds: int = 0,
                       tuple(float(x) for x in st.phase_ms) if time_phases else (), int(st.dp_rows_swept),
                       int(st.dp_launches),
                       tuple(int(x) for x in st.safeguard_objective) if safeguards and inst.mode == 0 else (),
-                      bool(st.used_top2), int(st.schedule))
+                      bool(st.used_top2), int(st.schedule), int(st.hw_queues))
 
 
 def pp_test_inject(kind: int, value: int):
@@ -312,10 +313,18 @@ def pp_dp_split(inst: Instance, batch: int, max_budget: int) -> dict:
     return {k: int(v) for k, v in zip(keys, out)}
 
 
-def pp_tune_dp(cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: bool = False,
+def pp_tune_dp(inst: Instance, cluster_ctas: int = 0, columns_per_thread: int = 0, force_flat: bool = False,
                no_prune: bool = False):
-    _check(_lib.pp_tune_dp(int(cluster_ctas), int(columns_per_thread), int(bool(force_flat)),
+    """Override this instance's DP launch shape (0 = automatic)."""
+    _check(_lib.pp_tune_dp(inst.handle, int(cluster_ctas), int(columns_per_thread), int(bool(force_flat)),
                            int(bool(no_prune))))
+
+
+def pp_dp_stack_bytes(inst: Instance) -> int:
+    """Bytes of skip-row stack scratch the instance holds (0 before any spilling launch)."""
+    out = ctypes.c_size_t(0)
+    _check(_lib.pp_dp_stack_bytes(inst.handle, ctypes.byref(out)))
+    return int(out.value)
 
 
 def pp_default_orders(inst: Instance, n_starts: int, stream=None) -> np.ndarray:
@@ -323,12 +332,6 @@ def pp_default_orders(inst: Instance, n_starts: int, stream=None) -> np.ndarray:
     out = np.zeros((int(n_starts), inst.W), np.int32)
     _check(_lib.pp_default_orders(inst.handle, int(n_starts), _host(out), _stream(stream)))
     return out
-
-
-def pp_probe_read(buf, iters: int, sink, stream=None):
-    """Read the CUDA tensor `buf` `iters` times (bandwidth probe); sink: 1-element int64 CUDA tensor."""
-    _check(_lib.pp_probe_read(_dev(buf), int(buf.numel() * buf.element_size()), int(iters), _dev(sink),
-                              _stream(stream)))
 
 
 def pp_safeguards(inst: Instance, stream=None):

@@ -1,8 +1,10 @@
 """In-tree build of libprefixplace.so for sm_103a (nvcc, no CMake).
 
-Each .cu file is compiled in parallel, then linked into one shared library
-next to this file.  The CUDA runtime is linked statically, so the library
-needs only the driver at run time and no torch symbols.
+Each .cu file under csrc/ is compiled in parallel, then linked into one
+shared library next to this file; the benchmark's bandwidth probe
+(probe/pp_probe.cu) becomes a library of its own, libpp_probe.so.  The CUDA
+runtime is linked statically, so the libraries need only the driver at run
+time and no torch symbols.
 """
 from __future__ import annotations
 
@@ -16,6 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libprefixplace.so")
+PROBE_SRC = os.path.join(HERE, "probe", "pp_probe.cu")
+PROBE_LIB = os.path.join(HERE, "libpp_probe.so")   # the benchmark's bandwidth probe, not the planner
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 
@@ -38,10 +42,12 @@ def _deps():
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+    if not os.path.exists(LIB) or not os.path.exists(PROBE_LIB):
         return False
     t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(f) <= t for f in _deps())
+    tp = os.path.getmtime(PROBE_LIB)
+    return all(os.path.getmtime(f) <= t for f in _deps()) and \
+        all(os.path.getmtime(f) <= tp for f in (PROBE_SRC, os.path.join(INCLUDE, "pp_probe.h")))
 
 
 def build(force: bool = False, verbose: bool = False, extra=()) -> str:
@@ -61,8 +67,18 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> str:
             print(r.stdout + r.stderr)
         return obj
 
+    def build_probe():
+        tmp = PROBE_LIB + f".tmp{os.getpid()}"
+        cmd = [nvcc, *ARCH, *FLAGS, *extra, "-shared", PROBE_SRC, "-o", tmp]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {PROBE_SRC}:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, PROBE_LIB)
+
     with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        probe = ex.submit(build_probe)
         objs = list(ex.map(compile_one, sources()))
+        probe.result()
     tmp = LIB + f".tmp{os.getpid()}"
     cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)

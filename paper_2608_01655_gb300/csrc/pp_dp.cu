@@ -1204,9 +1204,6 @@ static int max_smem_optin(const pp_instance *inst)
     return v;
 }
 
-// Geometry overrides set by pp_tune_dp (0 = automatic).
-static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0, g_tune_noprune = 0;
-
 // Split launch: measured on GB300 (152 SMs), the placement of clusters of 8
 // CTAs at one CTA per SM finds room for 15 of them; a 16th cluster then shares
 // SMs with other items and slows them and itself by ~25% per row.  When the
@@ -1216,7 +1213,7 @@ static int g_tune_cl = 0, g_tune_c = 0, g_tune_flat = 0, g_tune_noprune = 0;
 static void split_geometry(const pp_instance *inst, int batch, const void *fn, const cudaLaunchConfig_t &cfg0,
                            int smem_max, DpGeom *g)
 {
-    if (g_tune_cl > 0 || g_tune_c > 0 || batch < 2 || batch > 32 || g->CL < 2 || (g->CL & 1) || 2 * g->WPC > 16)
+    if (inst->tune_cl > 0 || inst->tune_c > 0 || batch < 2 || batch > 32 || g->CL < 2 || (g->CL & 1) || 2 * g->WPC > 16)
         return;
     int per_sm = 0;
     cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, inst->device);
@@ -1277,7 +1274,7 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     int per_item = inst->sm_count / std::max(batch, 1);
     per_item = std::max(1, std::min(8, per_item));
     int cl_hi = per_item;
-    if (g_tune_cl > 0) cl_hi = std::min(g_tune_cl, 8);
+    if (inst->tune_cl > 0) cl_hi = std::min(inst->tune_cl, 8);
     // Shape chosen by timing whole plans of the paper-scale workload at budgets
     // 128 to 4,096: 2 columns per thread (1 and 4 were slower) unless that
     // needs more than 32 warps per DP, then 4; a budget of at most 128 columns
@@ -1288,18 +1285,18 @@ static bool wave_geometry(const pp_instance *inst, int64_t k, int batch, DpGeom 
     // clusters that fit at one CTA per SM is split (split_geometry).
     int C = WMAX;
     bool one_warp = false;
-    if (g_tune_c > 0) {
-        C = std::max(std::min(g_tune_c, 8), WMAX);
+    if (inst->tune_c > 0) {
+        C = std::max(std::min(inst->tune_c, 8), WMAX);
     } else if (k <= 128) {
         while (32 * C < k) C *= 2;
-        one_warp = g_tune_cl <= 0;
+        one_warp = inst->tune_cl <= 0;
     } else {
         C = std::max(WMAX, 2);
         if ((k + 32 * C - 1) / (32 * C) > 32 && C < 4) C = 4;
         if ((k + 32 * C - 1) / (32 * C) > 128) C = 8;
     }
     const int64_t P = (k + 32 * C - 1) / (32 * C);     // warps per DP
-    if (g_tune_cl <= 0) cl_hi = (int)std::min<int64_t>(one_warp ? 1 : cl_hi, P);
+    if (inst->tune_cl <= 0) cl_hi = (int)std::min<int64_t>(one_warp ? 1 : cl_hi, P);
     for (int CL = cl_hi; CL >= 1; --CL) {
         const int WPC = (int)((P + CL - 1) / CL);
         if (WPC > 16) continue;
@@ -1356,7 +1353,7 @@ bool dp_geometry(const pp_instance *inst, int32_t max_budget, DpGeom *g, int bat
     int64_t k = max_budget;
     if (k > inst->total_weight) k = inst->total_weight;   // larger budgets change nothing
     if (k < 1) k = 1;
-    if (inst->max_weight <= 4 && inst->n > 0 && !g_tune_flat && wave_geometry(inst, k, batch, g)) return true;
+    if (inst->max_weight <= 4 && inst->n > 0 && !inst->tune_flat && wave_geometry(inst, k, batch, g)) return true;
     int C = 1;
     while ((int64_t)C * 1024 < k) C *= 2;
     if (C > 32) return false;
@@ -1434,7 +1431,7 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
         pc.numAttrs = 1;
         const int32_t *ord = inst->d_order, *nxt = inst->d_next, *wp = inst->d_wpre, *wm = inst->d_wave;
         const int2 *psp = inst->d_pspan;
-        const int pr = !g_tune_noprune, wv = g.wave, sd = inst->stack_depth;
+        const int pr = !inst->tune_noprune, wv = g.wave, sd = inst->stack_depth;
         int32_t *stt = inst->d_status;
         if (by_node)
             PP_CUDA(cudaLaunchKernelEx(&pc, k_prune<true>, inst->n, profit, ord, nxt, psp, wp, wm, item_active,
@@ -1601,16 +1598,17 @@ extern "C" pp_status pp_test_inject(int32_t kind, int32_t value)
     return PP_OK;
 }
 
-extern "C" pp_status pp_tune_dp(int32_t cluster_ctas, int32_t columns_per_thread, int32_t force_flat,
-                                int32_t no_prune)
+extern "C" pp_status pp_tune_dp(pp_instance *inst, int32_t cluster_ctas, int32_t columns_per_thread,
+                                int32_t force_flat, int32_t no_prune)
 {
+    if (!inst) return fail(PP_EINVAL, "null instance");
     if (cluster_ctas < 0 || cluster_ctas > 8 || columns_per_thread < 0 || columns_per_thread > 16 ||
         (columns_per_thread & (columns_per_thread - 1)) != 0)
         return fail(PP_EINVAL, "cluster_ctas must be 0..8 and columns_per_thread 0 or a power of two <= 16");
-    g_tune_cl = cluster_ctas;
-    g_tune_c = columns_per_thread;
-    g_tune_flat = force_flat != 0;
-    g_tune_noprune = no_prune != 0;
+    inst->tune_cl = cluster_ctas;
+    inst->tune_c = columns_per_thread;
+    inst->tune_flat = force_flat != 0;
+    inst->tune_noprune = no_prune != 0;
     return PP_OK;
 }
 
@@ -1709,6 +1707,13 @@ extern "C" pp_status pp_tree_dp_noalloc(pp_instance *inst, int32_t batch, const 
     return launch_dp_kernels(inst, batch, profit, true, budget, nullptr, g, best,
                              dp_work_split(bits, batch, inst->n, g.words), st, max_budget, scratch, L_glob,
                              nullptr);
+}
+
+extern "C" pp_status pp_dp_stack_bytes(const pp_instance *inst, size_t *out)
+{
+    if (!inst || !out) return fail(PP_EINVAL, "null pointer");
+    *out = inst->stack.ptr ? inst->stack.bytes : 0;
+    return PP_OK;
 }
 
 extern "C" pp_status pp_dp_rows_swept(const pp_instance *inst, int32_t batch, int32_t max_budget,

@@ -130,6 +130,8 @@ struct pp_instance {
     int64_t total_weight = 0;           // sum of chunk weights
     int32_t max_weight = 1;             // largest chunk weight
     int32_t trace_skips = 1;            // skips the traceback speculates per step beyond the first
+    // DP launch-shape overrides of this instance (pp_tune_dp; 0 = automatic)
+    int32_t tune_cl = 0, tune_c = 0, tune_flat = 0, tune_noprune = 0;
     std::vector<int32_t> h_order, h_next, h_budget, h_wpre, h_meta, h_wave;
     // device tables, preorder-indexed unless noted
     int32_t *d_order = nullptr;         // [n] position -> node id

@@ -479,6 +479,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         for (int c = 0; c < 3; ++c) stats->safeguard_objective[c] = so[c];
         stats->used_top2 = use_top2;
         stats->schedule = lockstep ? 1 : 2;
+        stats->hw_queues = hardware_queues();
         stats->phase_ms[0] = stats->phase_ms[1] = stats->phase_ms[2] = 0.f;
         // groups of four marks: before the marginals, the DP and the traceback, and after
         auto add = [&](const std::vector<cudaEvent_t> &v, size_t from, size_t to, float scale) {

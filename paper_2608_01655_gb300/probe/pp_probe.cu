@@ -1,10 +1,16 @@
-// Read-bandwidth probe for the benchmark's roofline denominators: every
-// thread streams 16-byte words of a buffer `iters` times.  With a buffer that
-// fits in L2 the loop measures L2 read bandwidth, with one far larger than
-// L2 it measures HBM read bandwidth.  Not part of the planner.
-#include "pp_internal.cuh"
+// Read-bandwidth probe for the benchmark's roofline denominators (a separate
+// library, libpp_probe.so, not part of the planner): every thread streams
+// 16-byte words of a buffer `iters` times.  With a buffer that fits in L2 the
+// loop measures L2 read bandwidth, with one far larger than L2 it measures
+// HBM read bandwidth.
+#include <cuda_runtime.h>
 
-namespace pp {
+#include <cstddef>
+#include <cstdint>
+
+#include "pp_probe.h"
+
+namespace {
 
 __global__ void __launch_bounds__(512) k_probe_read(const uint4 *__restrict__ p, size_t words, int iters,
                                                     unsigned long long *__restrict__ sink)
@@ -28,20 +34,16 @@ __global__ void __launch_bounds__(512) k_probe_read(const uint4 *__restrict__ p,
     if (acc == 0x9e3779b9u) atomicAdd(sink, 1ull);     // keeps the loads live
 }
 
-}  // namespace pp
+}  // namespace
 
-using namespace pp;
-
-extern "C" pp_status pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *sink, void *stream)
+extern "C" int pp_probe_read(const void *buf, size_t bytes, int32_t iters, uint64_t *sink, void *stream)
 {
-    if (!buf || !sink || iters < 0 || bytes % 16 || ((uintptr_t)buf & 15))
-        return fail(PP_EINVAL, "pp_probe_read: 16-byte aligned buffer, size a multiple of 16, iters >= 0");
-    if (bytes == 0 || iters == 0) return PP_OK;
+    if (!buf || !sink || iters < 0 || bytes % 16 || ((uintptr_t)buf & 15)) return 1;
+    if (bytes == 0 || iters == 0) return 0;
     int dev = 0, sms = 0;
-    PP_CUDA(cudaGetDevice(&dev));
-    PP_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    if (cudaGetDevice(&dev) != cudaSuccess) return 2;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 2;
     k_probe_read<<<sms * 4, 512, 0, (cudaStream_t)stream>>>(reinterpret_cast<const uint4 *>(buf), bytes / 16,
                                                             iters, reinterpret_cast<unsigned long long *>(sink));
-    PP_CUDA(cudaGetLastError());
-    return PP_OK;
+    return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

@@ -21,6 +21,25 @@ def my_starts(n_starts: int, rank: int, world: int) -> np.ndarray:
     return np.arange(rank, n_starts, world, dtype=np.int64)
 
 
+def total_starts(S: int, world: int, scaling: str) -> int:
+    """Starts of the whole job: weak scaling plans S starts per process
+    (S * world in all), strong scaling splits the S starts of one plan."""
+    if scaling not in ("weak", "strong"):
+        raise ValueError("scaling must be 'weak' or 'strong'")
+    return S * world if scaling == "weak" else S
+
+
+def rank_orders(default_orders, S: int, rank: int, world: int, scaling: str):
+    """The start orders this rank plans and their global start indices.
+
+    default_orders(total) -> [total][W] int32 must give the same orders on
+    every rank (pp_default_orders does: it depends on the instance only)."""
+    total = total_starts(S, world, scaling)
+    orders = np.asarray(default_orders(total), np.int32)
+    idx = my_starts(total, rank, world)
+    return orders[idx], idx
+
+
 @dataclass
 class ShardResult:
     objective: int

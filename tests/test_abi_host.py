@@ -22,22 +22,26 @@ def lib():
     return binding
 
 
-def _declared():
-    names = set()
-    for f in os.listdir(os.path.join(ROOT, "include")):
-        if f.endswith(".h"):
-            txt = open(os.path.join(ROOT, "include", f)).read()
-            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
-            names |= set(re.findall(r"\b(pp_\w+)\s*\(", txt))
-    return names
+def _declared(header):
+    txt = open(os.path.join(ROOT, "include", header)).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return set(re.findall(r"\b(pp_\w+)\s*\(", txt))
 
 
 def test_library_exports_every_declared_symbol(lib):
-    declared = _declared()
+    """Every entry point of include/prefixplace.h is exported by
+    libprefixplace.so, and the benchmark probe of include/pp_probe.h by
+    libpp_probe.so (and not by the planner's library)."""
+    headers = sorted(f for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h"))
+    assert headers == ["pp_probe.h", "prefixplace.h"]
+    declared = _declared("prefixplace.h")
     assert len(declared) >= 12
     so = ctypes.CDLL(lib.LIB_PATH)
     missing = [n for n in sorted(declared) if not hasattr(so, n)]
     assert not missing, missing
+    probe = ctypes.CDLL(ppbuild.PROBE_LIB)
+    assert _declared("pp_probe.h") == {"pp_probe_read"}
+    assert hasattr(probe, "pp_probe_read") and not hasattr(so, "pp_probe_read")
 
 
 def _create(lib, **kw):

@@ -106,11 +106,11 @@ def test_tree_dp_without_pruning(pp, oracle_lib):
         maxb = int(budgets.max())
         outs = []
         for no_prune in (True, False):
-            pp.pp_tune_dp(0, 0, False, no_prune)
+            pp.pp_tune_dp(ppi, 0, 0, False, no_prune)
             try:
                 outs.append(_dp_batch(pp, ppi, profits, budgets, maxb))
             finally:
-                pp.pp_tune_dp(0, 0, False, False)
+                pp.pp_tune_dp(ppi, 0, 0, False, False)
         for b in range(3):
             ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
             for best, chosen in outs:
@@ -438,7 +438,7 @@ def test_split_launch_matches_single_launch(pp, oracle_lib, B):
         bud = _dev(np.full(B, k), np.int32)
         outs = []
         for tune in [(0, 0), (8, 4)]:               # automatic (split), then one launch
-            pp.pp_tune_dp(*tune, False, False)
+            pp.pp_tune_dp(ppi, *tune, False, False)
             try:
                 best = torch.zeros(B, dtype=torch.int64, device="cuda")
                 bits = torch.zeros(pp.pp_dp_bits_size(ppi, B, k) // 4, dtype=torch.int32, device="cuda")
@@ -447,7 +447,7 @@ def test_split_launch_matches_single_launch(pp, oracle_lib, B):
                 pp.pp_traceback(ppi, bits, bud, k, chosen)
                 ppi.sync()
             finally:
-                pp.pp_tune_dp(0, 0, False, False)
+                pp.pp_tune_dp(ppi, 0, 0, False, False)
             outs.append((best.cpu().numpy(), bits.cpu().numpy(), chosen.cpu().numpy()))
     np.testing.assert_array_equal(outs[0][0], outs[1][0])
     np.testing.assert_array_equal(outs[0][1], outs[1][1])
@@ -487,11 +487,11 @@ def test_batch_of_16_with_stack_spill(pp, oracle_lib):
     budgets = rng.integers(k // 2, k + 1, size=B).astype(np.int32)
     outs = []
     for tune in [(0, 0), (8, 4)]:
-        pp.pp_tune_dp(*tune, False, False)
+        pp.pp_tune_dp(ppi, *tune, False, False)
         try:
             outs.append(_dp_batch(pp, ppi, profits, budgets, k))
         finally:
-            pp.pp_tune_dp(0, 0, False, False)
+            pp.pp_tune_dp(ppi, 0, 0, False, False)
     np.testing.assert_array_equal(outs[0][0], outs[1][0])
     np.testing.assert_array_equal(outs[0][1], outs[1][1])
     for b in (0, 7, 15):
@@ -519,6 +519,43 @@ def test_plan_per_start_streams_match_lockstep(pp, cfg):
     np.testing.assert_array_equal(a.per_start_sweeps, b.per_start_sweeps)
     np.testing.assert_array_equal(a.per_start_accepted, b.per_start_accepted)
     assert (a.dp_count, a.dp_cells, a.dp_rows_swept) == (b.dp_count, b.dp_cells, b.dp_rows_swept)
+
+
+def test_plan_16_starts_with_stack_spill(pp, oracle_lib):
+    """16 starts on a tree whose skip-row stack spills out of shared memory:
+    the per-start schedule (one stack slot per start, each start's DP CTAs
+    reserving more than half an SM) and lock step give the oracle's plan."""
+    rng = np.random.default_rng(1616)
+    parent = [-1]
+    spine = 0
+    for _ in range(70):                 # a spine whose nodes also have a leaf child: stack ~70 deep
+        nxt = len(parent)
+        parent.append(spine)
+        parent.append(spine)
+        spine = nxt
+    for _ in range(4000):
+        parent.append(int(rng.integers(len(parent))))
+    parent = np.asarray(parent, np.int32)
+    n, W, S, k = len(parent), 4, 16, 4096
+    base = wl.random_small(rng, n, W, 0, k_max=1, w_max=1, demand_max=30)
+    inst = wl.Instance("deep16", n, W, parent, np.ones(n, np.int32), base.demand,
+                       rng.integers(1000, 90000, size=(W, n)).astype(np.int64),
+                       rng.integers(500, 60000, size=(W, n)).astype(np.int64), 0,
+                       np.full(W, k, np.int32), S, 2)
+    o = oracle_lib.plan(oracle_lib.Problem.from_instance(inst), S, 2, safeguards=False)
+    with pp.Instance.from_workload(inst) as ppi:
+        order, nxt, depth = ppi.preorder()
+        assert pp.pp_dp_geometry(ppi, S, k)["stack_levels_smem"] < depth
+        a = pp.pp_plan_run(ppi, S, None, 2, safeguards=False, schedule=2)
+        assert pp.pp_dp_stack_bytes(ppi) > 0
+        b = pp.pp_plan_run(ppi, S, None, 2, safeguards=False, schedule=1)
+    assert (a.schedule, b.schedule) == (2, 1)
+    for g in (a, b):
+        assert g.objective == o.objective and g.best_start == o.best_start
+        np.testing.assert_array_equal(g.placement, o.placement)
+        np.testing.assert_array_equal(g.per_start_objective, o.per_start_objective)
+        np.testing.assert_array_equal(g.per_start_sweeps, o.per_start_sweeps)
+        np.testing.assert_array_equal(g.per_start_accepted, o.per_start_accepted)
 
 
 def test_plan_paper_scale_properties(pp, oracle_lib):

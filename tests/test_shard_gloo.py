@@ -99,6 +99,58 @@ def test_sharded_starts_match_one_process(oracle_lib, tmp_path, world, S, seed):
         np.testing.assert_array_equal(np.array(rec["placement"], np.uint8), full.placement)
 
 
+def _bench_worker(rank, world, port, seed, S, R, scaling, out_dir):
+    """The benchmark's rank logic (shard.rank_orders, then shard.exchange)
+    with the oracle as the planner."""
+    import datetime
+
+    import oracle
+    from paper_2608_01655_gb300 import shard
+
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world,
+                            timeout=datetime.timedelta(seconds=20))
+    inst = _instance(seed)
+    prob = oracle.Problem.from_instance(inst)
+    orders, idx = shard.rank_orders(lambda total: oracle.default_orders(prob, total), S, rank, world, scaling)
+    if len(idx):
+        r = oracle.plan(prob, len(idx), R, orders=orders, threads=1)
+        obj, start, placement = r.objective, int(idx[r.best_start]), r.placement
+    else:
+        obj, start, placement = 0, -1, np.zeros((inst.W, inst.n), np.uint8)
+    won = shard.exchange(obj, start, placement)
+    with open(os.path.join(out_dir, f"bench{rank}.json"), "w") as f:
+        json.dump({"objective": won.objective, "start": won.best_start, "planned": idx.tolist(),
+                   "placement": won.placement.astype(int).tolist()}, f)
+    dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world,scaling", [(2, "weak"), (3, "weak"), (2, "strong"), (3, "strong")])
+def test_bench_rank_logic_weak_and_strong(oracle_lib, tmp_path, world, scaling):
+    """Weak scaling: S starts per rank out of S * world default orders; strong
+    scaling: the S starts of one plan split over the ranks.  Either way the
+    ranks plan disjoint round-robin shares that cover every start, and the
+    exchanged winner equals one process planning all of those starts."""
+    S, R, seed = 4, 2, 5
+    port = _free_port()
+    ctx = mp.get_context("spawn")
+    procs = [ctx.Process(target=_bench_worker, args=(r, world, port, seed, S, R, scaling, str(tmp_path)))
+             for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+    assert [p.exitcode for p in procs] == [0] * world
+    total = S * world if scaling == "weak" else S
+    inst = _instance(seed)
+    prob = oracle_lib.Problem.from_instance(inst)
+    full = oracle_lib.plan(prob, total, R, orders=oracle_lib.default_orders(prob, total), threads=1)
+    recs = [json.load(open(tmp_path / f"bench{r}.json")) for r in range(world)]
+    assert sorted(sum((rec["planned"] for rec in recs), [])) == list(range(total))
+    for rec in recs:
+        assert rec["objective"] == full.objective and rec["start"] == full.best_start
+        np.testing.assert_array_equal(np.array(rec["placement"], np.uint8), full.placement)
+
+
 def test_lost_rank_is_reported(oracle_lib, tmp_path):
     """Rank 1 exits before the exchange; rank 0 gets an error within the
     process-group timeout instead of waiting forever."""

@@ -6,7 +6,9 @@ owned by its own caching allocator).  It keeps the skip-row stack levels that
 do not fit in shared memory in a fixed 16 MiB device array.  These checks
 compare it with pp_tree_dp on launches that really spill stack levels to that
 array, twice in a row (the second call must not be disturbed by what the
-first left in the array), and check the size limit.  This file sorts last so
+first left in the array), that the call leaves the instance without stack
+scratch of its own, that a batch pp_tree_dp would split runs as one launch
+with the same results, and check the size limit.  This file sorts last so
 that a run stopping at the first failure has run every other test before it.
 """
 import numpy as np
@@ -70,29 +72,63 @@ def test_noalloc_matches_tree_dp_twice(pp, oracle_lib, w_max, tune):
     rng = np.random.default_rng(900 + w_max)
     parent, weight = _deep_stack_tree(rng, 60, 3000, w_max)
     k = 4096
-    pp.pp_tune_dp(*tune)
-    try:
-        ppi = _instance(pp, parent, weight, k)
-        order, nxt, depth = ppi.preorder()
-        geo = pp.pp_dp_geometry(ppi, 2, k)
-        assert geo["stack_levels_smem"] < depth, (geo, depth)      # the fixed array is really used
-        budgets = np.array([k, k // 2 + 5], np.int32)
-        for call in range(2):
-            profits = rng.integers(0, 1000, size=(2, len(parent))).astype(np.int64)
-            profits[:, rng.random(len(parent)) < 0.3] = 0
-            ref = _run(pp, ppi, pp.pp_tree_dp, profits, budgets, k)
-            got = _run(pp, ppi, pp.pp_tree_dp_noalloc, profits, budgets, k)
-            if call == 0:                   # the spilling launch against the oracle itself
-                for b in range(2):
-                    ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
-                    assert int(ref[0][b]) == ob
-                    np.testing.assert_array_equal(ref[2][b], oc)
-            np.testing.assert_array_equal(got[0], ref[0])
-            np.testing.assert_array_equal(got[1], ref[1])
-            np.testing.assert_array_equal(got[2], ref[2])
-        ppi.close()
-    finally:
-        pp.pp_tune_dp(0, 0, False, False)
+    ppi = _instance(pp, parent, weight, k)
+    pp.pp_tune_dp(ppi, *tune)
+    order, nxt, depth = ppi.preorder()
+    geo = pp.pp_dp_geometry(ppi, 2, k)
+    assert geo["stack_levels_smem"] < depth, (geo, depth)      # the fixed array is really used
+    budgets = np.array([k, k // 2 + 5], np.int32)
+    for call in range(2):
+        profits = rng.integers(0, 1000, size=(2, len(parent))).astype(np.int64)
+        profits[:, rng.random(len(parent)) < 0.3] = 0
+        # on the fresh instance the allocation-free call runs first: it must
+        # leave the instance without stack scratch of its own
+        got = _run(pp, ppi, pp.pp_tree_dp_noalloc, profits, budgets, k)
+        if call == 0:
+            assert pp.pp_dp_stack_bytes(ppi) == 0
+        ref = _run(pp, ppi, pp.pp_tree_dp, profits, budgets, k)
+        assert pp.pp_dp_stack_bytes(ppi) > 0                 # pp_tree_dp spilled to its own scratch
+        if call == 0:                   # the spilling launch against the oracle itself
+            for b in range(2):
+                ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+                assert int(got[0][b]) == ob
+                np.testing.assert_array_equal(got[2][b], oc)
+        np.testing.assert_array_equal(got[0], ref[0])
+        np.testing.assert_array_equal(got[1], ref[1])
+        np.testing.assert_array_equal(got[2], ref[2])
+    ppi.close()
+
+
+def test_noalloc_runs_a_split_geometry_as_one_launch(pp, oracle_lib):
+    """A batch that pp_tree_dp splits into two concurrent launches (16 items:
+    15 on clusters of 8 CTAs, one on a narrower cluster beside them) runs as
+    one launch in the allocation-free call; values, decision bits and chosen
+    sets are the same.  (A split is only chosen when the wide clusters' stack
+    fits in less than half an SM's shared memory, so it never spills.)"""
+    if torch.cuda.get_device_properties(0).multi_processor_count != 152:
+        pytest.skip("the split is sized for a 152-SM GB300")
+    inst = wl.make(3)
+    rng = np.random.default_rng(961)
+    B, k = 16, int(inst.budget[0])
+    n = inst.n
+    ppi = _instance(pp, inst.parent, inst.weight, k)
+    assert pp.pp_dp_split(ppi, B, k)["wide_items"] > 0
+    profits = rng.integers(0, 10 ** 6, size=(B, n)).astype(np.int64)
+    profits[:, rng.random(n) < 0.5] = 0
+    budgets = rng.integers(k // 2, k + 1, size=B).astype(np.int32)
+    for call in range(2):
+        got = _run(pp, ppi, pp.pp_tree_dp_noalloc, profits, budgets, k)
+        ref = _run(pp, ppi, pp.pp_tree_dp, profits, budgets, k)
+        np.testing.assert_array_equal(got[0], ref[0])
+        np.testing.assert_array_equal(got[1], ref[1])
+        np.testing.assert_array_equal(got[2], ref[2])
+        if call == 0:
+            for b in (0, B - 1):
+                ob, oc = oracle_lib.rooted_dp(inst.parent, inst.weight, profits[b], int(budgets[b]))
+                assert int(got[0][b]) == ob
+                np.testing.assert_array_equal(got[2][b], oc)
+        profits = profits[::-1].copy()
+    ppi.close()
 
 
 def test_noalloc_rejects_oversized_launch(pp):
