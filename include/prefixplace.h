@@ -273,7 +273,8 @@ pp_status pp_dp_rows_swept(const pp_instance *inst, int32_t batch, int32_t max_b
 
 /*
  * pp_traceback -- recover each item's optimal parent-closed set from the
- * decision bits (Algorithm 1, "backtrack from D[1,k]"): start at position 0
+ * decision bits (Algorithm 1's backtracking, from the cell of the first row
+ * and the full budget): start at position 0
  * with j = k; "take" marks the chunk, j -= w_i and moves to i+1; "skip" moves
  * to next(i).  Among optimal sets this returns the lexicographically smallest
  * preorder indicator.
