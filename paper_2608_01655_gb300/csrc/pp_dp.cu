@@ -469,6 +469,9 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
 #pragma unroll
                     for (int u = 0; u < kSub; ++u) row(u, false, 0);   // no push or pop in these rows
                 }
+            } else if (cb8 == 0) {
+#pragma unroll
+                for (int u = 0; u < kSub; ++u) row(u, true, 2);        // stack operations, every skip row the top
             } else {
 #pragma unroll
                 for (int u = 0; u < kSub; ++u) row(u, true, 0);
@@ -1191,7 +1194,12 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
                     lvl = 0;
                 }
                 const int wq = wpre[rl[q]];
-                rm[q] = wave_pack(wq > 8 ? 8 : wq, s >= 0 && s == q - 1 ? kWaveCur : kWaveTop, flags, lvl);
+                // a row whose skip row is the row just computed reads it from the
+                // stack top when that row was pushed (the push made it the top):
+                // the same values, and sub-blocks without "cur" rows need no
+                // per-row choice of skip source
+                const bool cur = s >= 0 && s == q - 1 && lr_[q - 1] < 0;
+                rm[q] = wave_pack(wq > 8 ? 8 : wq, cur ? kWaveCur : kWaveTop, flags, lvl);
                 ex += dq[v];
             }
         }
