@@ -675,10 +675,12 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
 // lane l tests row t - l at the column reached after taking rows t..t-l+1, a
 // ballot gives the take-run, and the row that ends it is the skip.  A step
 // that leaves the tile (rows below it, or columns left of it) loads the next.
-// Helper warps of the walking warp's CTA follow its position through shared
-// memory and prefetch into L1 the tiles below it in its column band (this
-// tile's columns and the next ones to the left); the walk itself is
-// unchanged (~4% shorter walks in the paper-scale plan).
+// With unit chunk weights, helper warps of the walking warp's CTA follow its
+// position through shared memory and prefetch into L1 the tiles below it in
+// its column band (this tile's columns and the next ones to the left); the
+// walk itself is unchanged (~4% shorter walks in the paper-scale plan; with
+// chunk weights 1-2 the same prefetching made the source-dependent plan's
+// walks ~15% longer, so weighted walks go without it).
 // Planner mode (acc.mask != nullptr): the update is accepted in the greedy
 // pass, or in refinement iff D[0][k] > sum of p_h over the current T_h
 // (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
@@ -698,11 +700,10 @@ __device__ __forceinline__ void prefetch_l1(const void *p)
 // Helper warps (threads 32 .. 32 * (1 + kTraceHelpers) - 1): while the walker
 // works, prefetch the decision-bit lines of the kept-row blocks from its tile
 // down to kTraceAhead tiles below, for the 64 columns ending at its column,
-// nearest first, and the same rows of the skip targets, positions and suffix
-// weights.  walk[0], walk[1]: the walker's tile (first row, column); walk[2]:
+// nearest first, and the same rows of the skip targets and positions.  walk[0], walk[1]: the walker's tile (first row, column); walk[2]:
 // set when the walk is over.  Every address is inside the item's arrays.
 __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int nk, const int32_t *sk,
-                               const int32_t *rl, const int32_t *ws, int unit_weights, volatile int *walk)
+                               const int32_t *rl, volatile int *walk)
 {
     const int ht = threadIdx.x - 32, NH = 32 * kTraceHelpers;
     int last_r0 = -2, last_j0 = -1;
@@ -716,7 +717,8 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
         last_r0 = r0;
         last_j0 = j0;
         const int jl = j0 > 64 ? j0 - 63 : 1;
-        const int tlo = (jl - 1) / C, thi = (j0 - 1) / C;         // chain threads owning those columns
+        const int lgC = __ffs(C) - 1;                             // C is a power of two
+        const int tlo = (jl - 1) >> lgC, thi = (j0 - 1) >> lgC;   // chain threads owning those columns
         const int glo = tlo >> 5, ghi = min(thi >> 5, P - 1);
         const int ng = ghi - glo + 1;
         const int b_hi = min((r0 >> 5) + kTraceTileRows / 32 - 1, min(nblk, (nk + 31) >> 5) - 1);
@@ -724,7 +726,7 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
         const int nb = b_hi - b_lo + 1;
         const int lines = nb > 0 ? nb * ng * C : 0;
         for (int x = ht; x < lines; x += NH) {
-            const int c = x % C, gb = x / C;
+            const int c = x & (C - 1), gb = x >> lgC;
             const int gg = glo + gb % ng, b = b_hi - gb / ng;
             const int ln = gg == glo ? (tlo & 31) : 0;
             prefetch_l1(Bi + (((size_t)gg * nblk + b) * C + c) * 32 + ln);
@@ -733,12 +735,14 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
         for (int r = rlo + 32 * ht; r < rhi; r += 32 * NH) {
             prefetch_l1(sk + r);
             prefetch_l1(rl + r);
-            if (!unit_weights) prefetch_l1(ws + r);
         }
     }
 }
 
-template <int SKIPS>
+// BYNODE: the ABI mode (chosen bytes by node id, acc.mask == nullptr);
+// otherwise the planner's accept-and-update mode.  A template parameter, so
+// the planner's walk carries no trace of the ABI mode's node-id loads.
+template <int SKIPS, bool BYNODE>
 __global__ void __launch_bounds__(256)
 k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
@@ -779,8 +783,8 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     const int32_t *ws = w.wsuf + (size_t)item * (n + 1);
     const int nk = w.nkept[item];
     if (threadIdx.x >= 32) {
-        if (threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0)
-            trace_prefetch(Bi, nblk, C, P, nk, sk, rl, ws, unit_weights, walk);
+        if (threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0 && unit_weights)
+            trace_prefetch(Bi, nblk, C, P, nk, sk, rl, walk);
         return;
     }
     const int lane = threadIdx.x;
@@ -790,9 +794,10 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     }
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
+    const int lgC = __ffs(C) - 1;
     auto word_at = [&](int blk, int col) -> uint32_t {       // bits of rows blk*32.. at column col >= 1
         const int q = col - 1;
-        const int tt = q / C, c = q - tt * C;
+        const int tt = q >> lgC, c = q & (C - 1);             // C is a power of two
         return Bi[(((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31)];
     };
     int t = nk - 1;                 // row of position 0 (the first root): swept last
@@ -813,6 +818,9 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
             wv[x] = (colx >= 1 && r0 + 32 * x < nk) ? word_at((r0 >> 5) + x, colx) : 0u;
             skv[x] = r < nk ? sk[r] : -1;
             rlv[x] = r < nk ? rl[r] : 0;
+            // ABI mode writes chosen[] by node id: fetch the rows' node ids with
+            // the tile rather than one dependent load per step
+            if (BYNODE && r < nk) rlv[x] = order[rlv[x]];
             wsv[x] = (!unit_weights && r < nk) ? ws[r] : 0;
         }
         const int wstop = unit_weights ? 0 : ws[min(r0 + kTraceTileRows, nk)];
@@ -869,8 +877,8 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
                 tnext = more ? sk1 : tnext;
             }
             if (lane < L) {
-                if (M) atomicOr(M + pos, hbit);               // a reduction: the walk does not wait on it
-                else chosen[(size_t)item * n + order[pos]] = 1;
+                if (BYNODE) chosen[(size_t)item * n + pos] = 1;   // pos: the row's node id here
+                else atomicOr(M + pos, hbit);                 // a reduction: the walk does not wait on it
             }
             if (L == 32) {                                    // 32 takes: continue after the last
                 j = __shfl_sync(kFull, coln, 31);
@@ -1620,14 +1628,22 @@ pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, con
                            cudaStream_t st)
 {
     if (batch <= 0 || inst->n == 0) return PP_OK;
+    if (g.C < 1 || (g.C & (g.C - 1))) return fail(PP_EINVAL, "columns per thread must be a power of two");
     AcceptArgs a;
     if (acc) a = *acc;
-    if (inst->trace_skips >= 3)
-        k_traceback<3><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
-                                              inst->d_order, chosen, a);
-    else
-        k_traceback<1><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, inst->max_weight <= 1, item_budget,
-                                              inst->d_order, chosen, a);
+    const int unit = inst->max_weight <= 1;
+    const bool bynode = a.mask == nullptr;
+    if (inst->trace_skips >= 3) {
+        if (bynode) k_traceback<3, true><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
+                                                                 inst->d_order, chosen, a);
+        else k_traceback<3, false><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
+                                                           inst->d_order, chosen, a);
+    } else {
+        if (bynode) k_traceback<1, true><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
+                                                                 inst->d_order, chosen, a);
+        else k_traceback<1, false><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
+                                                           inst->d_order, chosen, a);
+    }
     PP_CUDA(cudaGetLastError());
     return PP_OK;
 }
