@@ -346,9 +346,12 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             // lap bit of this pass over the ring
             const uint64_t lap = (uint64_t)((r0 / kRing) & 1) << 63;
             const uint64_t *sl = my_ring + (size_t)(r0 & (kRing - 1)) * WMAX;
+            // the slots' values (read by the wait below); the first warp has no
+            // previous warp and reads zeros (column 0 of every row is 0)
             uint64_t sv[WMAX == 1 ? kSub : 1];
 #pragma unroll
-            for (int u = 0; u < (WMAX == 1 ? kSub : 1); ++u) sv[u] = 0;
+            for (int u = 0; u < (WMAX == 1 ? kSub : 1); ++u)
+                if (!has_prev) sv[u] = 0;
             const bool need_ack = has_next && r0 + kSub + 1 > kRing && ack_seen < (uint32_t)(r0 + kSub + 1 - kRing);
             if (has_prev || need_ack) {
                 const uint32_t need = (uint32_t)(r0 + kSub + 1 - kRing);
@@ -433,7 +436,11 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
                     if (publish) nx_gen[(r0 & (kRing - 1)) * WMAX + u * WMAX + q] = (uint64_t)cur[C - WMAX + q] | lap;
                 // skip-row stack (warp-uniform masks): push (the new row becomes
                 // the top), reload the new top after a pop, or reset it to the zero row
-                if (STACK && ((stk8 >> u) & 1u)) {
+                // the masks are warp-uniform; with unit weights, saying so with a
+                // vote lets the compiler drop the reconvergence of every row's
+                // branch in the stack path (DP phase of the paper-scale plan
+                // 160.1 -> 156.2 ms; the weighted kernels ran slower with it)
+                if (STACK && (WMAX == 1 ? __any_sync(kFull, (stk8 >> u) & 1u) : ((stk8 >> u) & 1u) != 0)) {
                     if ((pb >> u) & 1u) {
                         const int lvl = (int)((uint32_t)my_m[s8 + u] >> 16);
 #pragma unroll
