@@ -821,18 +821,11 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
         return !(ident && (wave || (wmeta[i] & kWaveStackOps) == 0));
     };
     slice(n, lo, hi);
-    int kmine = 0, wmine = 0;
-    for (int r = lo + t; r < hi; r += T)
-        if (keep(r)) {
-            kmine += 1;
-            wmine += wpre[n - 1 - r];
-        }
+    int kmine = 0;
+    for (int r = lo + t; r < hi; r += T) kmine += keep(r);
     block_exclusive_scan(kmine, &total, sh);
     int kcarry = cluster_exclusive_scan(total, &total, &slot, bcast);
     const int nk = total;
-    block_exclusive_scan(wmine, &total, sh);
-    int wtot;
-    cluster_exclusive_scan(total, &wtot, &slot, bcast);   // weight of all kept rows
     for (int base = lo; base < hi; base += tile) {
         bool kp[V];
         int kc = 0;
@@ -872,10 +865,11 @@ k_prune(int32_t n, const int64_t *__restrict__ profit, const int32_t *__restrict
     int64_t *rp = w.rowp + (size_t)item * n;
     int32_t *rm = w.rowm + (size_t)item * n;
     slice(nk, lo, hi);
-    wmine = 0;
+    int wmine = 0;
     for (int q = lo + t; q < hi; q += T) wmine += wpre[rl[q]];
     block_exclusive_scan(wmine, &total, sh);
-    int wcarry = cluster_exclusive_scan(total, &total, &slot, bcast);
+    int wtot;                                             // weight of all kept rows
+    int wcarry = cluster_exclusive_scan(total, &wtot, &slot, bcast);
     for (int base = lo; base < hi; base += tile) {
         int wq[V], wl = 0;
 #pragma unroll
