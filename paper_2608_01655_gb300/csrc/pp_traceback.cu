@@ -74,7 +74,9 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
         const int lines = nb > 0 ? nb * ng * C : 0;
         for (int x = ht; x < lines; x += NH) {
             const int c = x & (C - 1), gb = x >> lgC;
-            const int gg = glo + gb % ng, b = b_hi - gb / ng;
+            // 64 columns span at most three chain warps: no run-time division
+            const int bq = ng == 1 ? gb : ng == 2 ? gb >> 1 : gb / 3;
+            const int gg = glo + (gb - bq * ng), b = b_hi - bq;
             const int ln = gg == glo ? (tlo & 31) : 0;
             prefetch_l1(Bi + (((size_t)gg * nblk + b) * C + c) * 32 + ln);
         }
