@@ -65,7 +65,10 @@ typedef struct {
     int32_t *orders_used;          /* [n_starts][W] host, out: the start orders */
     int32_t best_start;            /* out: index of the returned candidate (>= n_starts:
                                       safeguard best_start - n_starts) */
-    int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded) */
+    int32_t dp_count;              /* out: tree DPs executed (inactive starts excluded; with
+                                      default orders and n_starts > 1 every start's first
+                                      greedy update walks the standalone-score DP of its
+                                      worker, which is the same DP, so it is not run again) */
     int64_t dp_cells;              /* out: sum over executed DPs of n * k_h (Eq. 9 cells) */
     int32_t kernel_launches;       /* out: kernels launched by this call */
     int64_t dp_rows_swept;         /* out: rows the DPs actually swept (pruned sweep), summed */

@@ -229,6 +229,9 @@ struct AcceptArgs {
     int32_t *accepted = nullptr;        // [batch] accepted-update counter
     uint32_t *mask = nullptr;           // [batch][n] holder masks (preorder)
     int greedy = 0;                     // 1: always accept (WorkerGreedy pass)
+    // optional [batch]: item b walks the decision bits (and pruned-sweep data)
+    // of DP item bits_item[b] of the workspace instead of item b
+    const int32_t *bits_item = nullptr;
 };
 pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, const DpGeom &g,
                            const int32_t *item_budget, uint8_t *chosen, const AcceptArgs *acc,

@@ -256,8 +256,38 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         t2.oldbit = reinterpret_cast<uint8_t *>(base + b3);
         PP_CUDA(cudaMemsetAsync(base, 0, b2, st));                 // v1 = v2 = 0: no holders yet
         PP_CUDA(cudaMemsetAsync(t2.l1, 0xFF, tw, st));             // l1 = -1
+        PP_CUDA(cudaMemsetAsync(t2.oldbit, 0, (size_t)S * n, st)); // nobody holds anything yet
     }
     PP_CUDA(cudaMemsetAsync(pb.improved, 0, 4 * S, st));
+    // The first greedy update of every start runs against an empty placement,
+    // so its marginals and its DP are exactly the standalone-score DP of its
+    // worker, computed above for the default orders: the start walks those
+    // decision bits (one batched traceback, item s reading DP item pi_s[0] of
+    // the standalone workspace) instead of running that DP again.
+    const bool reuse = standalone_cells > 0;
+    int64_t reused_cells = 0;
+    if (reuse)
+        for (int32_t x = 0; x < S; ++x) reused_cells += (int64_t)n * inst->h_budget[ord[(size_t)x * W]];
+    auto first_from_standalone = [&]() -> pp_status {
+        pp_status r;
+        if ((r = mark())) return r;
+        if ((r = mark())) return r;       // no marginal pass
+        if ((r = mark())) return r;       // no DP
+        AcceptArgs a;
+        a.worker = pb.work;               // step 0: pi_s[0]
+        a.best = pb.best;
+        a.oldsum = pb.oldsum;
+        a.active = pb.active;
+        a.improved = pb.improved;
+        a.accepted = pb.accepted;
+        a.mask = pb.mask;
+        a.greedy = 1;
+        a.bits_item = pb.work;
+        if ((r = launch_traceback(inst, S, work_w, gw, pb.kbud, nullptr, &a, st))) return r;
+        if ((r = mark())) return r;
+        launches += 1;
+        return PP_OK;
+    };
     // lock step unless asked for per-start streams, or (automatic) unless every
     // start's stream gets a hardware queue of its own: streams that share a
     // queue wait on one another's launches, which costs more than lock step
@@ -302,10 +332,16 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         };
 
         // WorkerGreedy pass
-        for (int32_t t = 0; t < W; ++t)
+        for (int32_t t = 0; t < W; ++t) {
+            if (t == 0 && reuse) {
+                if ((s = first_from_standalone())) return s;
+                prev_wk = pb.work;        // top-2: step 0's change is folded in at step 1
+                continue;
+            }
             if ((s = step(t, 1))) return s;
-        dp_count += S * W;
-        cells += (int64_t)S * n * sumk;
+        }
+        dp_count += S * W - (reuse ? S : 0);
+        cells += (int64_t)S * n * sumk - reused_cells;
 
         // coordinate refinement
         std::vector<int32_t> act(S, 1);
@@ -346,6 +382,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
             PP_CUDA(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, inst->device));
             g1.smem = std::max(g1.smem, (size_t)std::min(per_sm / 2, optin));
         }
+        if (reuse && (s = first_from_standalone())) return s;     // on the caller's stream, before the fork
         PP_CUDA(cudaEventRecord(inst->plan_fork, st));
         for (int x = 0; x < NS; ++x) PP_CUDA(cudaStreamWaitEvent(inst->plan_streams[x], inst->plan_fork, 0));
         std::vector<const int32_t *> prev(S, nullptr);
@@ -362,6 +399,10 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         const size_t N = (size_t)std::max(n, 1);
         for (int q = 0; q < W * (1 + R); ++q) {
             const int pass = q / W, t = q % W;
+            if (q == 0 && reuse) {
+                for (int x = 0; x < S; ++x) prev[x] = pb.work + x;    // top-2: folded in at step 1
+                continue;
+            }
             for (int x = 0; x < S; ++x) {
                 cudaStream_t sx = inst->plan_streams[x % NS];
                 const int32_t *wk = pb.work + (size_t)t * B + x;
@@ -428,9 +469,9 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
         // executed updates, from the sweeps each start ran (the greedy pass always runs)
         int64_t swsum = 0;
         for (int32_t x = 0; x < S; ++x) swsum += sw[x];
-        dp_count += (int)(S * W + swsum * W);
-        cells += ((int64_t)S + swsum) * n * sumk;
-        dp_launches += (int32_t)((W * (S + swsum) + S / 2) / S);
+        dp_count += (int)(S * W + swsum * W) - (reuse ? S : 0);
+        cells += ((int64_t)S + swsum) * n * sumk - reused_cells;
+        dp_launches += (int32_t)((W * (S + swsum) - (reuse ? S : 0) + S / 2) / S);
     }
     int32_t bs = 0;
     for (int32_t x = 1; x < S; ++x)
@@ -498,7 +539,7 @@ pp_status plan_impl(pp_instance *inst, int32_t S, const int32_t *orders, int32_t
             add(ev, 0, ev.size(), 1.f);
         } else {
             // the standalone-score step (on the caller's stream), then the mean over starts
-            add(ev, 0, standalone_cells ? 4 : 0, 1.f);
+            add(ev, 0, standalone_cells ? 8 : 0, 1.f);      // with the batched first traceback
             for (const auto &v : sev) add(v, 0, v.size(), 1.f / (float)S);
         }
     }

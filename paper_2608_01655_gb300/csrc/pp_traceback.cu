@@ -125,12 +125,13 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     __syncthreads();
     volatile int *walk = s_walk;
     const int32_t kq = item_budget[item];
+    const int bi = acc.bits_item ? acc.bits_item[item] : item;   // the DP item whose bits this walks
     const int nblk = (n + 31) / 32;
-    const uint32_t *Bi = w.bits + (size_t)item * P * (size_t)nblk * C * 32;
-    const int32_t *rl = w.rowlist + (size_t)item * n;
-    const int32_t *sk = w.skip + (size_t)item * n;
-    const int32_t *ws = w.wsuf + (size_t)item * (n + 1);
-    const int nk = w.nkept[item];
+    const uint32_t *Bi = w.bits + (size_t)bi * P * (size_t)nblk * C * 32;
+    const int32_t *rl = w.rowlist + (size_t)bi * n;
+    const int32_t *sk = w.skip + (size_t)bi * n;
+    const int32_t *ws = w.wsuf + (size_t)bi * (n + 1);
+    const int nk = w.nkept[bi];
     if (threadIdx.x >= 32) {
         if (threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0 && unit_weights)
             trace_prefetch(Bi, nblk, C, P, nk, sk, rl, walk);

@@ -252,7 +252,11 @@ def test_plan_parity_workloads(pp, oracle_lib, cfg):
         g = pp.pp_plan_run(ppi, inst.starts, None, inst.rounds)
     o = oracle_lib.plan(prob, inst.starts, inst.rounds)
     _compare_plans(g, o)
-    assert g.dp_cells == o.cells
+    # with default orders and several starts, every start's first greedy update
+    # (an empty placement) walks the standalone-score DP of its worker instead
+    # of running it again: the oracle evaluates those cells, the GPU does not
+    reused = sum(inst.n * int(inst.budget[g.orders[x][0]]) for x in range(inst.starts)) if inst.starts > 1 else 0
+    assert g.dp_cells == o.cells - reused
 
 
 def test_plan_top2_marginals(pp, oracle_lib):
