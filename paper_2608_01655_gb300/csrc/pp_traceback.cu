@@ -16,28 +16,46 @@ constexpr unsigned kFull = 0xffffffffu;
 // at i = n or j = 0.  In kept-row order a take always moves from kept index t
 // to t - 1 (the next kept row in preorder, since a pruned interior is all
 // "skip"), and a skip moves to skip[t].  The walk is monotone in t and j, so
-// one warp reads it tile by tile: a tile is 64 kept rows x 32 columns, whose
-// decision bits are 64 words (one word holds 32 rows of one column), loaded
-// together with the tile's skip targets, positions and suffix weights in one
-// round of independent loads.  Inside the tile every step is register work:
-// lane l tests row t - l at the column reached after taking rows t..t-l+1, a
-// ballot gives the take-run, and the row that ends it is the skip.  A step
-// that leaves the tile (rows below it, or columns left of it) loads the next.
+// one warp reads it tile by tile.  A tile is 64 kept rows x 64 columns in
+// shared memory: per column one 64-bit word of take bits (two of the DP's
+// 32-row words), and per row its skip target, preorder position and suffix
+// weight, brought in with asynchronous 4-byte copies.  Inside the tile a step
+// is: lane l reads the bit of row t - l at the column reached after taking
+// rows t..t-l+1, a warp min-reduction gives the first lane that does not take
+// (the take-run's end), and that lane's row is the skip, whose target (and,
+// speculatively, the target's own skip in the same column word) comes from
+// the same tile.  The rows a step takes form a run of tile rows: they are
+// gathered in a 64-bit mask and marked when the walk leaves the tile, so no
+// global memory operation sits on the steps' chain of dependent operations.
+// The copies are software-pipelined: on entering a tile the walker starts
+// those of the tile below it, anchored at its entry column, into the other
+// of two buffers; a walk that leaves downwards within 64 columns (skips are
+// short; ~15 columns per tile on the paper-scale trees) finds it on chip, and
+// any other exit copies its tile on demand.
 // With unit chunk weights, helper warps of the walking warp's CTA follow its
 // position through shared memory and prefetch into L1 the tiles below it in
-// its column band (this tile's columns and the next ones to the left); the
-// walk itself is unchanged (~4% shorter walks in the paper-scale plan; with
-// chunk weights 1-2 the same prefetching made the source-dependent plan's
-// walks ~15% longer, so weighted walks go without it).
+// its column band, for the demand copies.
 // Planner mode (acc.mask != nullptr): the update is accepted in the greedy
 // pass, or in refinement iff D[0][k] > sum of p_h over the current T_h
 // (equivalent to G(T_-h, T'_h) > G(T) by Prop. 1); an accepted update
 // replaces bit h of the holder masks by the traced set.
 // ===========================================================================
-constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (a multiple of 32)
+constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (one 64-bit word per column)
+constexpr int kTraceTileCols = 64;       // columns per traceback tile
 constexpr int kTraceHelpers = 3;         // prefetching warps beside the walking one
 constexpr int kTraceAhead = 4;           // tiles below the walker's that they prefetch
 constexpr uint32_t kTracePollLimit = 1u << 22;   // polls of the walker's position (~0.4 s)
+
+// 4-byte asynchronous global -> shared copy; with `read` false nothing is
+// read and the destination is zero-filled
+__device__ __forceinline__ void cp_async4(void *dst, const void *src, bool read)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
+                 "l"(__cvta_generic_to_global(src)), "r"(read ? 4 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 __device__ __forceinline__ void prefetch_l1(const void *p)
 {
@@ -88,12 +106,22 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
     }
 }
 
+// One traceback tile in shared memory: kept rows r0..r0+63 at the 64 columns
+// a, a-1, .., a-63 (column index c = a - column).
+struct TraceTile {
+    uint64_t bits[kTraceTileCols];       // bit lr of bits[c]: take at row r0 + lr, column a - c
+    int32_t skip[kTraceTileRows];        // skip target (kept index) of row r0 + lr, -1 past n
+    int32_t pos[kTraceTileRows];         // preorder position of row r0 + lr (node id in the ABI mode)
+    int32_t ws[kTraceTileRows + 1];      // suffix weight at row r0 + lr (lr = 64: at r0 + 64)
+};
+
 // BYNODE: the ABI mode (chosen bytes by node id, acc.mask == nullptr);
-// otherwise the planner's accept-and-update mode.  A template parameter, so
-// the planner's walk carries no trace of the ABI mode's node-id loads.
-template <int SKIPS, bool BYNODE>
+// otherwise the planner's accept-and-update mode.  UNIT: every chunk weight
+// is 1 (and helper warps prefetch for the walker).  Template parameters, so
+// that each walk carries no trace of the other modes.
+template <int SKIPS, bool BYNODE, bool UNIT>
 __global__ void __launch_bounds__(256)
-k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
+k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
             const int32_t *__restrict__ item_budget, const int32_t *__restrict__ order,
             uint8_t *__restrict__ chosen, AcceptArgs acc)
 {
@@ -133,7 +161,7 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     const int32_t *ws = w.wsuf + (size_t)bi * (n + 1);
     const int nk = w.nkept[bi];
     if (threadIdx.x >= 32) {
-        if (threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0 && unit_weights)
+        if (UNIT && threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0)
             trace_prefetch(Bi, nblk, C, P, nk, sk, rl, walk);
         return;
     }
@@ -145,108 +173,127 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad, int unit_weights,
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
     const int lgC = __ffs(C) - 1;
-    auto word_at = [&](int blk, int col) -> uint32_t {       // bits of rows blk*32.. at column col >= 1
+    auto word_index = [&](int blk, int col) -> size_t {    // word of rows blk*32.. at column col >= 1
         const int q = col - 1;
         const int tt = q >> lgC, c = q & (C - 1);             // C is a power of two
-        return Bi[(((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31)];
+        return (((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31);
+    };
+    // start the copies of the tile of rows r0.. at columns a, a-1, ..: lane l
+    // copies columns a-l and a-32-l and rows r0+l and r0+32+l; what lies left
+    // of column 1 or at rows >= nk is zero-filled (never read as valid)
+    __shared__ TraceTile s_tile[2];
+    auto stage = [&](TraceTile &T, int r0, int a) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int c = lane + 32 * h, col = a - c;
+            uint32_t *dst = reinterpret_cast<uint32_t *>(&T.bits[c]);
+#pragma unroll
+            for (int b = 0; b < 2; ++b) {
+                const bool rd = col >= 1 && r0 + 32 * b < nk;
+                cp_async4(dst + b, rd ? (const void *)&Bi[word_index((r0 >> 5) + b, col)] : (const void *)Bi, rd);
+            }
+            const int r = r0 + c;
+            const bool in = r < nk;
+            cp_async4(&T.skip[c], in ? (const void *)(sk + r) : (const void *)Bi, in);
+            cp_async4(&T.pos[c], in ? (const void *)(rl + r) : (const void *)Bi, in);
+            if (!UNIT) cp_async4(&T.ws[c], in ? (const void *)(ws + r) : (const void *)Bi, in);
+        }
+        if (!UNIT && lane == 0) cp_async4(&T.ws[kTraceTileRows], ws + min(r0 + kTraceTileRows, nk), true);
+        cp_async_commit();
     };
     int t = nk - 1;                 // row of position 0 (the first root): swept last
-    constexpr int TB = kTraceTileRows / 32;                   // 32-row blocks per tile
+    int pr0 = -1, pa = 0;           // the tile copied ahead: rows pr0.., columns pa, pa-1, ..
     for (int guard = 0; guard <= 2 * n + 2 && t >= 0 && j > 0; ++guard) {
-        // ---- load the tile holding (t, j): rows r0..r0+TB*32-1, columns j0-31..j0
-        const int r0 = t & ~(kTraceTileRows - 1), j0 = j;
+        // ---- the tile holding (t, j), from the copy made ahead when it is that one
+        const int r0 = t & ~(kTraceTileRows - 1);
+        const int slot = (r0 / kTraceTileRows) & 1;
+        TraceTile &T = s_tile[slot];
+        cp_async_wait_all();
+        __syncwarp();                         // every lane's copies, and the last tile's reads, are done
+        int a = pa;
+        if (r0 != pr0 || j <= pa - kTraceTileCols) {
+            a = j;
+            stage(T, r0, a);
+            cp_async_wait_all();
+            __syncwarp();
+        }
+        if (BYNODE) {                         // ABI mode marks chosen[] by node id
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+                if (r0 + lane + 32 * h < nk) T.pos[lane + 32 * h] = order[T.pos[lane + 32 * h]];
+            __syncwarp();
+        }
         if (lane == 0) {                      // where the helpers prefetch next
-            walk[1] = j0;
+            walk[1] = j;
             walk[0] = r0;
         }
-        const int colx = j0 - lane;
-        uint32_t wv[TB];
-        int skv[TB], rlv[TB], wsv[TB];
-#pragma unroll
-        for (int x = 0; x < TB; ++x) {
-            const int r = r0 + 32 * x + lane;
-            wv[x] = (colx >= 1 && r0 + 32 * x < nk) ? word_at((r0 >> 5) + x, colx) : 0u;
-            skv[x] = r < nk ? sk[r] : -1;
-            rlv[x] = r < nk ? rl[r] : 0;
-            // ABI mode writes chosen[] by node id: fetch the rows' node ids with
-            // the tile rather than one dependent load per step
-            if (BYNODE && r < nk) rlv[x] = order[rlv[x]];
-            wsv[x] = (!unit_weights && r < nk) ? ws[r] : 0;
-        }
-        const int wstop = unit_weights ? 0 : ws[min(r0 + kTraceTileRows, nk)];
-        // a register of block lr / 32 of the lane lr % 32 (every lane calls it)
-        auto pick = [&](const auto &v, int lr, int from) {
-            int out = 0;
-#pragma unroll
-            for (int x = 0; x < TB; ++x) {
-                const int y = __shfl_sync(kFull, (int)v[x], from);
-                out = (lr >> 5) == x ? y : out;
-            }
-            return out;
-        };
-        // suffix weight of kept row r in r0..r0+TB*32
-        auto wsat = [&](int r) -> int {
-            const int lr = r - r0;
-            const int y = pick(wsv, lr, lr & 31);
-            return lr >= kTraceTileRows ? wstop : y;
-        };
-        // ---- walk inside the tile
-        while (t >= r0 && j > 0 && j > j0 - 32) {
-            const int row = t - lane;
-            const int lr = (row - r0) & (kTraceTileRows - 1);
+        // ---- copy the tile below ahead, anchored at this column: a walk that
+        // leaves downwards (skips are short: ~15 columns per 64-row tile on the
+        // paper-scale trees) finds it on chip
+        pr0 = r0 - kTraceTileRows;
+        pa = j;
+        if (pr0 >= 0) stage(s_tile[slot ^ 1], pr0, pa);
+        // ---- walk inside the tile: lane l tests row t-l at the column reached
+        // after taking rows t..t-l+1.  The rows a step takes are a run of tile
+        // rows, gathered in `taken` and marked when the walk leaves the tile,
+        // off the steps' chain of dependent operations.
+        uint64_t taken = 0;
+        bool inside = t >= r0 && a - j < kTraceTileCols;      // j > 0 here
+        while (inside) {
+            const int lt = t - r0, lr = lt - lane;
             int col, coln;
-            if (unit_weights) {
+            if (UNIT) {
                 col = j - lane;
                 coln = col - 1;
             } else {
-                const int wt = wsat(t + 1), wr = wsat(row + 1), wr0 = wsat(row);
-                col = j - (wr - wt);
-                coln = j - (wr0 - wt);
+                const int wt = T.ws[lt + 1];
+                col = j - (T.ws[max(lr + 1, 0)] - wt);
+                coln = j - (T.ws[max(lr, 0)] - wt);
             }
-            const bool valid = row >= r0 && col >= 1 && col > j0 - 32;
-            const uint32_t word = (uint32_t)pick(wv, lr, (j0 - col) & 31);
-            const bool take = valid && ((word >> (lr & 31)) & 1u);
-            const uint32_t tm = __ballot_sync(kFull, take);
-            const int L = tm == kFull ? 32 : __ffs(~tm) - 1;    // rows t..t-L+1 are taken
-            const int pos = pick(rlv, lr, lr & 31);
-            const int skr = pick(skv, lr, lr & 31);
+            const int ci = a - col;
+            const bool valid = lr >= 0 && col >= 1 && ci < kTraceTileCols;
+            const int lrm = lr & (kTraceTileRows - 1);
+            const uint64_t word = T.bits[min(max(ci, 0), kTraceTileCols - 1)];
+            const int skr = T.skip[lrm];
+            const bool take = valid && ((word >> lrm) & 1ull);
+            // the first lane that does not take (32: all take): rows t..t-L+1 are taken
+            const int L = (int)__reduce_min_sync(kFull, take ? 32u : (unsigned)lane);
             // speculation for the lane that ends the take-run: its skip lands
-            // on row skr at the same column; while that row is in the tile and
-            // is skipped as well, the walk goes on to its skip target in the
-            // same step, up to SKIPS times (skips often come in pairs: with one,
-            // ~35% fewer steps at the paper-scale workload; trees with wide
-            // fan-out have longer runs and use three)
+            // on row skr at the same column (the same word); while that row is
+            // in the tile and is skipped as well, the walk goes on to its skip
+            // target in the same step, up to SKIPS times (skips often come in
+            // pairs; trees with wide fan-out have longer chains and use three)
             int tnext = skr;
             bool more = true;
 #pragma unroll
             for (int d = 0; d < SKIPS; ++d) {
-                const int lr1 = (tnext - r0) & (kTraceTileRows - 1);
-                const uint32_t word1 = (uint32_t)pick(wv, lr1, (j0 - col) & 31);
-                const int sk1 = pick(skv, lr1, lr1 & 31);
-                more = more && tnext >= r0 && !((word1 >> (lr1 & 31)) & 1u);
-                tnext = more ? sk1 : tnext;
+                const int l1 = tnext - r0;
+                more = more && l1 >= 0 && !((word >> (l1 & (kTraceTileRows - 1))) & 1ull);
+                const int s1 = T.skip[l1 & (kTraceTileRows - 1)];
+                tnext = more ? s1 : tnext;
             }
-            if (lane < L) {
+            if (L > 0) taken |= ((2ull << (L - 1)) - 1) << (lt - L + 1);
+            // next state: after 32 takes, row t-32 at the column after them;
+            // else lane L's row is skipped (to tnext) when it lies in the tile,
+            // and otherwise the walk leaves the tile at (t-L, its column)
+            const int colL = UNIT ? j - L : __shfl_sync(kFull, L == 32 ? coln : col, L == 32 ? 31 : L);
+            const int skL = __shfl_sync(kFull, tnext, L & 31);
+            const bool all = L == 32;
+            const bool inL = !all && lt - L >= 0 && colL >= 1 && a - colL < kTraceTileCols;
+            t = all ? t - 32 : inL ? skL : t - L;       // skL = -1: past n
+            j = colL;
+            inside = (all || inL) && t >= r0 && j > 0 && a - j < kTraceTileCols;
+        }
+        // ---- mark the taken rows: lane l the tile rows l and l+32
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+            if ((taken >> (lane + 32 * h)) & 1ull) {
+                const int pos = T.pos[lane + 32 * h];
                 if (BYNODE) chosen[(size_t)item * n + pos] = 1;   // pos: the row's node id here
                 else atomicOr(M + pos, hbit);                 // a reduction: the walk does not wait on it
             }
-            if (L == 32) {                                    // 32 takes: continue after the last
-                j = __shfl_sync(kFull, coln, 31);
-                t -= 32;
-                continue;
-            }
-            const int vL = __shfl_sync(kFull, (int)valid, L);
-            const int colL = __shfl_sync(kFull, col, L);
-            const int skL = __shfl_sync(kFull, tnext, L);
-            j = colL;
-            if (vL) {
-                t = skL;                // row t-L is skipped (and maybe next(t-L)): -1 = past n
-            } else {
-                t -= L;                                       // (t-L, colL) lies outside the tile
-                break;
-            }
-        }
     }
+    cp_async_wait_all();                      // no copy outlives the block
     if (lane == 0) walk[2] = 1;               // the helpers stop
 }
 
@@ -261,16 +308,16 @@ pp_status launch_traceback(pp_instance *inst, int batch, const DpWork &work, con
     if (acc) a = *acc;
     const int unit = inst->max_weight <= 1;
     const bool bynode = a.mask == nullptr;
-    if (inst->trace_skips >= 3) {
-        if (bynode) k_traceback<3, true><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
-                                                                 inst->d_order, chosen, a);
-        else k_traceback<3, false><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
-                                                           inst->d_order, chosen, a);
+    const int skips = inst->trace_skips >= 3 ? 3 : 1;
+    auto go = [&](auto kern) {
+        kern<<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, item_budget, inst->d_order, chosen, a);
+    };
+    if (skips == 3) {
+        if (bynode) unit ? go(k_traceback<3, true, true>) : go(k_traceback<3, true, false>);
+        else unit ? go(k_traceback<3, false, true>) : go(k_traceback<3, false, false>);
     } else {
-        if (bynode) k_traceback<1, true><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
-                                                                 inst->d_order, chosen, a);
-        else k_traceback<1, false><<<batch, 256, 0, st>>>(inst->n, work, g.C, g.P, g.kpad, unit, item_budget,
-                                                           inst->d_order, chosen, a);
+        if (bynode) unit ? go(k_traceback<1, true, true>) : go(k_traceback<1, true, false>);
+        else unit ? go(k_traceback<1, false, true>) : go(k_traceback<1, false, false>);
     }
     PP_CUDA(cudaGetLastError());
     return PP_OK;
