@@ -273,7 +273,9 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
     const bool publish = has_next && lane == 31 && g != g_drop_publish_warp;   // this lane stores
     const bool lane0 = lane == 0;
 
-    uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + lane;
+    // decision bits in block pairs: the words of 32-row blocks 2b and 2b+1
+    // of one column sit side by side (one 8-byte word per 64 rows)
+    uint32_t *Bw = bits + ((size_t)item * P + g) * (size_t)nblk * C * 32 + 2 * lane;
     int64_t *gst = gstack + (((size_t)item * L_glob) * CL + cr) * (size_t)C * NT;
     int64_t *const my_gst = gst + threadIdx.x;
     // this warp's shared-memory stack levels: a column's word of a level sits
@@ -498,7 +500,7 @@ k_tree_dp_wave(int32_t n, int32_t nblk, const int64_t *__restrict__ rowp,
             }
         }
 #pragma unroll
-        for (int c = 0; c < C; ++c) Bw[((size_t)blk * C + c) * 32] = wbits[c];
+        for (int c = 0; c < C; ++c) Bw[((size_t)(blk >> 1) * C + c) * 64 + (blk & 1)] = wbits[c];
     }
 
     asm volatile("cp.async.wait_all;" ::: "memory");   // nothing in flight into this CTA's shared memory
@@ -564,8 +566,8 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
     int32_t *sm = sw + 2 * kMetaRows;
     int64_t *gst = gstack + (size_t)item * L_glob * kpad;
     const int64_t *Pp = profit + (size_t)item * n;
-    const int nblk = (n + 31) / 32;
-    uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)nblk * C * 32 + lane;
+    const int nblk = (n + 63) / 64 * 2;                      // 32-row blocks, in pairs
+    uint32_t *Bw = bits + ((size_t)item * P + warp) * (size_t)nblk * C * 32 + 2 * lane;
     const int nrows = rowlist ? nkept[item] : n;
     const int32_t *rows = rowlist ? rowlist + (size_t)item * n : nullptr;
     uint32_t wbits[C];
@@ -635,7 +637,7 @@ k_tree_dp_flat(int32_t n, const int32_t *__restrict__ rowlist, const int32_t *__
         if ((r & 31) == 31 || r == nrows - 1) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
-                Bw[((size_t)(r >> 5) * C + c) * 32] = wbits[c];
+                Bw[((size_t)(r >> 6) * C + c) * 64 + ((r >> 5) & 1)] = wbits[c];
                 wbits[c] = 0;
             }
         }
@@ -984,14 +986,14 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 size_t dp_work_bytes(int batch, int n, int words)
 {
-    const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
+    const size_t nb = (size_t)(n + 63) / 64 * 64, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
     return align256(B * nb * words * 4) + 4 * align256(B * N * 4) + 2 * align256(B * (N + 1) * 4) +
            align256(B * 4) + align256(B * N * 8);
 }
 
 DpWork dp_work_split(void *base, int batch, int n, int words)
 {
-    const size_t nb = (size_t)(n + 31) / 32 * 32, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
+    const size_t nb = (size_t)(n + 63) / 64 * 64, B = (size_t)std::max(batch, 1), N = (size_t)std::max(n, 1);
     char *p = reinterpret_cast<char *>(base);
     DpWork w;
     w.bits = reinterpret_cast<uint32_t *>(p);
@@ -1016,7 +1018,7 @@ DpWork dp_work_split(void *base, int batch, int n, int words)
 
 DpWork dp_work_item(const DpWork &w, int item, int n, int words)
 {
-    const size_t nb = (size_t)(n + 31) / 32 * 32, N = (size_t)std::max(n, 1), it = (size_t)item;
+    const size_t nb = (size_t)(n + 63) / 64 * 64, N = (size_t)std::max(n, 1), it = (size_t)item;
     DpWork o;
     o.bits = w.bits + it * nb * words;
     o.rowlist = w.rowlist + it * N;
@@ -1299,7 +1301,7 @@ static pp_status launch_dp_kernels(pp_instance *inst, int batch, const int64_t *
     const int32_t *nkept = work.nkept;
     if (g.wave) {
         int32_t n = inst->n;
-        int32_t nblk = (n + 31) / 32;
+        int32_t nblk = (n + 63) / 64 * 2;                    // 32-row blocks, in pairs
         const int64_t *rowp = work.rowp;
         const int32_t *rowm = work.rowm;
         int32_t *status = inst->d_status;

@@ -1,9 +1,10 @@
 // Traceback of the tree DP's decision bits (Algorithm 1's backtracking,
 // Theorem 1: at most n visited states) and, in the planner, the accept-and-
 // update step fused into it (Section IV-C, Prop. 1).  The bits are those
-// pp_dp.cu's kernels write: for chain warp g, lane and column offset c, the
-// word (((item * P + g) * nblk + r / 32) * C + c) * 32 + lane holds the take
-// decisions of kept rows r (sweep order) at column (g * 32 + lane) * C + c + 1.
+// pp_dp.cu's kernels write, in block pairs: for chain warp g, lane and column
+// offset c, the 8-byte word ((item * P + g) * nblk / 2 + r / 64) * C + c) * 32
+// + lane holds the take decisions of kept rows r (sweep order, 64 rows, bit
+// r % 64) at column (g * 32 + lane) * C + c + 1.
 #include "pp_internal.cuh"
 
 namespace pp {
@@ -46,12 +47,18 @@ constexpr int kTraceHelpers = 3;         // prefetching warps beside the walking
 constexpr int kTraceAhead = 4;           // tiles below the walker's that they prefetch
 constexpr uint32_t kTracePollLimit = 1u << 22;   // polls of the walker's position (~0.4 s)
 
-// 4-byte asynchronous global -> shared copy; with `read` false nothing is
-// read and the destination is zero-filled
+// 4- and 8-byte asynchronous global -> shared copies; with `read` false
+// nothing is read and the destination is zero-filled
 __device__ __forceinline__ void cp_async4(void *dst, const void *src, bool read)
 {
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
                  "l"(__cvta_generic_to_global(src)), "r"(read ? 4 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async8(void *dst, const void *src, bool read)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
+                 "l"(__cvta_generic_to_global(src)), "r"(read ? 8 : 0)
                  : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
@@ -67,7 +74,7 @@ __device__ __forceinline__ void prefetch_l1(const void *p)
 // down to kTraceAhead tiles below, for the 64 columns ending at its column,
 // nearest first, and the same rows of the skip targets and positions.  walk[0], walk[1]: the walker's tile (first row, column); walk[2]:
 // set when the walk is over.  Every address is inside the item's arrays.
-__device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int nk, const int32_t *sk,
+__device__ void trace_prefetch(const uint64_t *Bi, int npair, int C, int P, int nk, const int32_t *sk,
                                const int32_t *rl, volatile int *walk)
 {
     const int ht = threadIdx.x - 32, NH = 32 * kTraceHelpers;
@@ -86,19 +93,19 @@ __device__ void trace_prefetch(const uint32_t *Bi, int nblk, int C, int P, int n
         const int tlo = (jl - 1) >> lgC, thi = (j0 - 1) >> lgC;   // chain threads owning those columns
         const int glo = tlo >> 5, ghi = min(thi >> 5, P - 1);
         const int ng = ghi - glo + 1;
-        const int b_hi = min((r0 >> 5) + kTraceTileRows / 32 - 1, min(nblk, (nk + 31) >> 5) - 1);
-        const int b_lo = max(0, (r0 >> 5) - kTraceAhead * (kTraceTileRows / 32));
+        const int b_hi = min(r0 >> 6, min(npair, (nk + 63) >> 6) - 1);      // 64-row block pairs
+        const int b_lo = max(0, (r0 >> 6) - kTraceAhead);
         const int nb = b_hi - b_lo + 1;
-        const int lines = nb > 0 ? nb * ng * C : 0;
+        const int lines = nb > 0 ? nb * ng * C * 2 : 0;                    // a pair row spans two lines
         for (int x = ht; x < lines; x += NH) {
-            const int c = x & (C - 1), gb = x >> lgC;
+            const int hh = x & 1, c = (x >> 1) & (C - 1), gb = x >> (lgC + 1);
             // 64 columns span at most three chain warps: no run-time division
             const int bq = ng == 1 ? gb : ng == 2 ? gb >> 1 : gb / 3;
             const int gg = glo + (gb - bq * ng), b = b_hi - bq;
-            const int ln = gg == glo ? (tlo & 31) : 0;
-            prefetch_l1(Bi + (((size_t)gg * nblk + b) * C + c) * 32 + ln);
+            const int ln = min((gg == glo ? (tlo & 31) : 0) + 16 * hh, 31);
+            prefetch_l1(Bi + (((size_t)gg * npair + b) * C + c) * 32 + ln);
         }
-        const int rlo = b_lo * 32, rhi = min(nk, (b_hi + 1) * 32);
+        const int rlo = b_lo * 64, rhi = min(nk, (b_hi + 1) * 64);
         for (int r = rlo + 32 * ht; r < rhi; r += 32 * NH) {
             prefetch_l1(sk + r);
             prefetch_l1(rl + r);
@@ -154,15 +161,15 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
     volatile int *walk = s_walk;
     const int32_t kq = item_budget[item];
     const int bi = acc.bits_item ? acc.bits_item[item] : item;   // the DP item whose bits this walks
-    const int nblk = (n + 31) / 32;
-    const uint32_t *Bi = w.bits + (size_t)bi * P * (size_t)nblk * C * 32;
+    const int npair = (n + 63) / 64;                          // 64-row block pairs per chain warp
+    const uint64_t *Bi = reinterpret_cast<const uint64_t *>(w.bits) + (size_t)bi * P * (size_t)npair * C * 32;
     const int32_t *rl = w.rowlist + (size_t)bi * n;
     const int32_t *sk = w.skip + (size_t)bi * n;
     const int32_t *ws = w.wsuf + (size_t)bi * (n + 1);
     const int nk = w.nkept[bi];
     if (threadIdx.x >= 32) {
         if (UNIT && threadIdx.x < 32 * (1 + kTraceHelpers) && kq > 0)
-            trace_prefetch(Bi, nblk, C, P, nk, sk, rl, walk);
+            trace_prefetch(Bi, npair, C, P, nk, sk, rl, walk);
         return;
     }
     const int lane = threadIdx.x;
@@ -173,25 +180,21 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
     if (kq <= 0) return;
     int32_t j = kq < kpad ? kq : kpad;
     const int lgC = __ffs(C) - 1;
-    auto word_index = [&](int blk, int col) -> size_t {    // word of rows blk*32.. at column col >= 1
+    auto word_index = [&](int bp, int col) -> size_t {     // 8-byte word of rows bp*64.. at column col >= 1
         const int q = col - 1;
         const int tt = q >> lgC, c = q & (C - 1);             // C is a power of two
-        return (((size_t)(tt >> 5) * nblk + blk) * C + c) * 32 + (tt & 31);
+        return (((size_t)(tt >> 5) * npair + bp) * C + c) * 32 + (tt & 31);
     };
     // start the copies of the tile of rows r0.. at columns a, a-1, ..: lane l
-    // copies columns a-l and a-32-l and rows r0+l and r0+32+l; what lies left
-    // of column 1 or at rows >= nk is zero-filled (never read as valid)
+    // copies columns a-l and a-32-l (one 8-byte word each) and rows r0+l and
+    // r0+32+l; what lies left of column 1 or at rows >= nk is zero-filled or
+    // stale, and never read as valid
     __shared__ TraceTile s_tile[2];
     auto stage = [&](TraceTile &T, int r0, int a) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             const int c = lane + 32 * h, col = a - c;
-            uint32_t *dst = reinterpret_cast<uint32_t *>(&T.bits[c]);
-#pragma unroll
-            for (int b = 0; b < 2; ++b) {
-                const bool rd = col >= 1 && r0 + 32 * b < nk;
-                cp_async4(dst + b, rd ? (const void *)&Bi[word_index((r0 >> 5) + b, col)] : (const void *)Bi, rd);
-            }
+            cp_async8(&T.bits[c], col >= 1 ? (const void *)&Bi[word_index(r0 >> 6, col)] : (const void *)Bi, col >= 1);
             const int r = r0 + c;
             const bool in = r < nk;
             cp_async4(&T.skip[c], in ? (const void *)(sk + r) : (const void *)Bi, in);
