@@ -17,10 +17,10 @@ constexpr unsigned kFull = 0xffffffffu;
 // at i = n or j = 0.  In kept-row order a take always moves from kept index t
 // to t - 1 (the next kept row in preorder, since a pruned interior is all
 // "skip"), and a skip moves to skip[t].  The walk is monotone in t and j, so
-// one warp reads it tile by tile.  A tile is 64 kept rows x 64 columns in
-// shared memory: per column one 64-bit word of take bits (two of the DP's
-// 32-row words), and per row its skip target, preorder position and suffix
-// weight, brought in with asynchronous 4-byte copies.  Inside the tile a step
+// one warp reads it tile by tile.  A tile is 64 kept rows x 96 columns in
+// shared memory: per column one 64-bit word of take bits (a block pair of the
+// DP's), and per row its skip target, preorder position and suffix weight,
+// brought in with asynchronous 8- and 4-byte copies.  Inside the tile a step
 // is: lane l reads the bit of row t - l at the column reached after taking
 // rows t..t-l+1, a warp min-reduction gives the first lane that does not take
 // (the take-run's end), and that lane's row is the skip, whose target (and,
@@ -30,9 +30,9 @@ constexpr unsigned kFull = 0xffffffffu;
 // global memory operation sits on the steps' chain of dependent operations.
 // The copies are software-pipelined: on entering a tile the walker starts
 // those of the tile below it, anchored at its entry column, into the other
-// of two buffers; a walk that leaves downwards within 64 columns (skips are
-// short; ~15 columns per tile on the paper-scale trees) finds it on chip, and
-// any other exit copies its tile on demand.
+// of two buffers; a walk that leaves downwards within 96 columns of that
+// anchor (skips are short; ~15 columns per tile on the paper-scale trees)
+// finds it on chip, and any other exit copies its tile on demand.
 // With unit chunk weights, helper warps of the walking warp's CTA follow its
 // position through shared memory and prefetch into L1 the tiles below it in
 // its column band, for the demand copies.
@@ -42,7 +42,7 @@ constexpr unsigned kFull = 0xffffffffu;
 // replaces bit h of the holder masks by the traced set.
 // ===========================================================================
 constexpr int kTraceTileRows = 64;       // kept rows per traceback tile (one 64-bit word per column)
-constexpr int kTraceTileCols = 64;       // columns per traceback tile
+constexpr int kTraceTileCols = 96;       // columns per traceback tile (a multiple of 32)
 constexpr int kTraceHelpers = 3;         // prefetching warps beside the walking one
 constexpr int kTraceAhead = 4;           // tiles below the walker's that they prefetch
 constexpr uint32_t kTracePollLimit = 1u << 22;   // polls of the walker's position (~0.4 s)
@@ -113,8 +113,8 @@ __device__ void trace_prefetch(const uint64_t *Bi, int npair, int C, int P, int 
     }
 }
 
-// One traceback tile in shared memory: kept rows r0..r0+63 at the 64 columns
-// a, a-1, .., a-63 (column index c = a - column).
+// One traceback tile in shared memory: kept rows r0..r0+63 at the columns
+// a, a-1, .., a-kTraceTileCols+1 (column index c = a - column).
 struct TraceTile {
     uint64_t bits[kTraceTileCols];       // bit lr of bits[c]: take at row r0 + lr, column a - c
     int32_t skip[kTraceTileRows];        // skip target (kept index) of row r0 + lr, -1 past n
@@ -186,15 +186,14 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
         return (((size_t)(tt >> 5) * npair + bp) * C + c) * 32 + (tt & 31);
     };
     // start the copies of the tile of rows r0.. at columns a, a-1, ..: lane l
-    // copies columns a-l and a-32-l (one 8-byte word each) and rows r0+l and
-    // r0+32+l; what lies left of column 1 or at rows >= nk is zero-filled or
-    // stale, and never read as valid
+    // copies rows r0+l and r0+32+l and columns a-l, a-32-l, .. (one 8-byte
+    // word each); what lies left of column 1 or at rows >= nk is zero-filled
+    // or stale, and never read as valid
     __shared__ TraceTile s_tile[2];
     auto stage = [&](TraceTile &T, int r0, int a) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int c = lane + 32 * h, col = a - c;
-            cp_async8(&T.bits[c], col >= 1 ? (const void *)&Bi[word_index(r0 >> 6, col)] : (const void *)Bi, col >= 1);
+            const int c = lane + 32 * h;
             const int r = r0 + c;
             const bool in = r < nk;
             cp_async4(&T.skip[c], in ? (const void *)(sk + r) : (const void *)Bi, in);
@@ -202,6 +201,11 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
             if (!UNIT) cp_async4(&T.ws[c], in ? (const void *)(ws + r) : (const void *)Bi, in);
         }
         if (!UNIT && lane == 0) cp_async4(&T.ws[kTraceTileRows], ws + min(r0 + kTraceTileRows, nk), true);
+#pragma unroll
+        for (int c = lane; c < kTraceTileCols; c += 32) {
+            const int col = a - c;
+            cp_async8(&T.bits[c], col >= 1 ? (const void *)&Bi[word_index(r0 >> 6, col)] : (const void *)Bi, col >= 1);
+        }
         cp_async_commit();
     };
     int t = nk - 1;                 // row of position 0 (the first root): swept last
@@ -220,11 +224,13 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
             cp_async_wait_all();
             __syncwarp();
         }
-        if (BYNODE) {                         // ABI mode marks chosen[] by node id
+        // the preorder positions of this lane's two tile rows, for marking
+        // (node ids in the ABI mode, which marks chosen[] by node id)
+        int posv[2];
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
-                if (r0 + lane + 32 * h < nk) T.pos[lane + 32 * h] = order[T.pos[lane + 32 * h]];
-            __syncwarp();
+        for (int h = 0; h < 2; ++h) {
+            posv[h] = T.pos[lane + 32 * h];
+            if (BYNODE && r0 + lane + 32 * h < nk) posv[h] = order[posv[h]];
         }
         if (lane == 0) {                      // where the helpers prefetch next
             walk[1] = j;
@@ -232,7 +238,9 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
         }
         // ---- copy the tile below ahead, anchored at this column: a walk that
         // leaves downwards (skips are short: ~15 columns per 64-row tile on the
-        // paper-scale trees) finds it on chip
+        // paper-scale trees) finds it on chip (tile width: 96 columns took the
+        // weighted plan's walks 15.1 -> 14.6 ms and left the unit-weight ones
+        // as they were, against 64)
         pr0 = r0 - kTraceTileRows;
         pa = j;
         if (pr0 >= 0) stage(s_tile[slot ^ 1], pr0, pa);
@@ -291,9 +299,8 @@ k_traceback(int32_t n, DpWork w, int C, int P, int kpad,
 #pragma unroll
         for (int h = 0; h < 2; ++h)
             if ((taken >> (lane + 32 * h)) & 1ull) {
-                const int pos = T.pos[lane + 32 * h];
-                if (BYNODE) chosen[(size_t)item * n + pos] = 1;   // pos: the row's node id here
-                else atomicOr(M + pos, hbit);                 // a reduction: the walk does not wait on it
+                if (BYNODE) chosen[(size_t)item * n + posv[h]] = 1;
+                else atomicOr(M + posv[h], hbit);             // a reduction: the walk does not wait on it
             }
     }
     cp_async_wait_all();                      // no copy outlives the block
