@@ -142,6 +142,59 @@ def test_tree_dp_multi_column_tiles(pp, oracle_lib, n, wmax, kmax):
         np.testing.assert_array_equal(chosen[b], oc)
 
 
+def _tile_crossing_trees(rng):
+    """Trees whose walks cross the traceback's tiles in every way: a long chain
+    (take-runs of 32 along the diagonal, column exits), a broom of chains from
+    one root (skips over whole chains, far past the tile below), and a
+    caterpillar (a spine whose nodes carry three leaves each: many single
+    skips between takes)."""
+    chain = np.arange(-1, 2999, dtype=np.int32)
+    broom = [-1]
+    for _ in range(24):
+        broom.append(0)
+        broom.extend(range(len(broom) - 1, len(broom) + 148))
+    broom = np.asarray(broom, np.int32)
+    cater = [-1]
+    spine = 0
+    for _ in range(600):
+        for _ in range(3):
+            cater.append(spine)
+        cater.append(spine)
+        spine = len(cater) - 1
+    cater = np.asarray(cater, np.int32)
+    return [("chain", chain), ("broom", broom), ("caterpillar", cater)]
+
+
+@pytest.mark.parametrize("wmax", [1, 4])
+def test_traceback_tile_crossings(pp, oracle_lib, wmax):
+    """Optimum and traced set, bit-exact, on walks that leave their tile by
+    rows, by columns and by skips far past the tile below, with budgets around
+    the 32-row run, 64-row tile and 96-column tile boundaries."""
+    rng = np.random.default_rng(4242 + wmax)
+    for name, parent in _tile_crossing_trees(rng):
+        n = len(parent)
+        weight = rng.integers(1, wmax + 1, size=n).astype(np.int32)
+        ppi = _tree_instance(pp, parent, weight)
+        B = 6
+        profits = rng.integers(1, 50, size=(B, n)).astype(np.int64)
+        if name == "broom":                    # whole chains cheap: the walk skips them
+            heads = np.flatnonzero(parent == 0)
+            for b in range(0, B, 2):
+                for h in heads[rng.random(len(heads)) < 0.5]:
+                    profits[b, h:h + 149] = 1
+        profits[1] = rng.integers(0, 3, size=n) * 40      # ties and zeros
+        tw = int(weight.sum())
+        budgets = np.array([min(tw, 2 * n // 3), 31, 32, 64, 96, min(tw, 97 + int(rng.integers(0, 400)))],
+                           np.int32)
+        maxb = int(budgets.max())
+        best, chosen = _dp_batch(pp, ppi, profits, budgets, maxb)
+        for b in range(B):
+            ob, oc = oracle_lib.rooted_dp(parent, weight, profits[b], int(budgets[b]))
+            assert best[b] == ob, (name, b)
+            np.testing.assert_array_equal(chosen[b], oc, err_msg=f"{name} item {b}")
+        ppi.close()
+
+
 @pytest.mark.parametrize("mode", [0, 1])
 def test_marginals_and_objective(pp, oracle_lib, mode):
     """Eq. 10 / Eq. 7 marginals and Eq. 4 / Eq. 6 objectives, bit-exact."""
