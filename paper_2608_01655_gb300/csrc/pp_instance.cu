@@ -5,6 +5,8 @@
 #include <cstdio>
 #include <cstring>
 #include <new>
+#include <thread>
+#include <vector>
 
 #include "pp_internal.cuh"
 
@@ -280,16 +282,59 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     //  sum Lambda * w: objectives (Eq. 4, Eq. 6), marginals and DP values;
     //  sum Lambda:     the Popularity safeguard's DP values (profit Lambda);
     //  sum w:          the epoch update's one-time cost (at most one w per (m, b)).
-    __int128 total = 0, sum_demand = 0, sum_recompute = 0;
-    for (size_t x = 0; x < Wn; ++x) {
-        if (demand[x] < 0 || recompute[x] < 0) return fail(PP_EINVAL, "negative demand or recompute cost");
-        total += (__int128)demand[x] * (__int128)recompute[x];
-        sum_demand += demand[x];
-        sum_recompute += recompute[x];
+    // The cost arrays are checked before anything is allocated, on up to 16
+    // host threads when they are large (the source-dependent transfer costs
+    // are W^2 n values: 102 MB at the paper-scale workload).
+    // Unsigned 128-bit sums (a negative value sets bit 63 of the OR and fails
+    // before its sum is used); the products and the running sum of products
+    // are capped at 2^63, above the 2^62 limit, so nothing wraps.
+    using u128 = unsigned __int128;
+    const u128 cap = (u128)1 << 63;
+    struct Part {
+        u128 total = 0, demand = 0, recompute = 0;
+        uint64_t dr_bits = 0, t_bits = 0;          // OR of the values: bit 63 = a negative one
+    };
+    const size_t work = Wn + tn;
+    const unsigned hw = std::max(1u, std::thread::hardware_concurrency());
+    const int nth = work < ((size_t)1 << 20) ? 1 : (int)std::min<unsigned>(hw, 16);
+    std::vector<Part> parts(nth);
+    auto check = [&](int q) {
+        Part &P = parts[q];
+        const size_t a = Wn * q / nth, b = Wn * (q + 1) / nth;
+        for (size_t x = a; x < b; ++x) {
+            const uint64_t dv = (uint64_t)demand[x], rv = (uint64_t)recompute[x];
+            P.dr_bits |= dv | rv;
+            const u128 pr = (u128)dv * rv;
+            P.total = std::min<u128>(P.total + std::min(pr, cap), cap);
+            P.demand += dv;
+            P.recompute += rv;
+        }
+        const size_t c = tn * q / nth, d = tn * (q + 1) / nth;
+        uint64_t tb = 0;
+        for (size_t x = c; x < d; ++x) tb |= (uint64_t)transfer[x];
+        P.t_bits = tb;
+    };
+    if (nth == 1) {
+        check(0);
+    } else {
+        std::vector<std::thread> pool;
+        pool.reserve(nth - 1);
+        for (int q = 1; q < nth; ++q) pool.emplace_back(check, q);
+        check(0);
+        for (auto &th : pool) th.join();
     }
-    for (size_t x = 0; x < tn; ++x)
-        if (transfer[x] < 0) return fail(PP_EINVAL, "negative transfer cost");
-    const __int128 lim = (__int128)1 << 62;
+    u128 total = 0, sum_demand = 0, sum_recompute = 0;
+    uint64_t dr_bits = 0, t_bits = 0;
+    for (const Part &P : parts) {
+        total = std::min<u128>(total + P.total, cap);
+        sum_demand += P.demand;
+        sum_recompute += P.recompute;
+        dr_bits |= P.dr_bits;
+        t_bits |= P.t_bits;
+    }
+    if (dr_bits >> 63) return fail(PP_EINVAL, "negative demand or recompute cost");
+    if (t_bits >> 63) return fail(PP_EINVAL, "negative transfer cost");
+    const u128 lim = (u128)1 << 62;
     if (total > lim) return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
     if (sum_demand > lim) return fail(PP_EOVERFLOW, "sum of demand exceeds 2^62");
     if (sum_recompute > lim) return fail(PP_EOVERFLOW, "sum of recompute costs exceeds 2^62");

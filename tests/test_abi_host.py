@@ -91,6 +91,30 @@ def test_create_validation_is_host_side(lib):
     assert st != lib.PP_EOVERFLOW
 
 
+def test_create_validation_large_and_extreme(lib):
+    """The cost arrays' checks hold where they are split over host threads
+    (W^2 n transfer costs above 2^20 values) and where the sum of products
+    would leave every 128-bit range (products near 2^126)."""
+    top = np.full((2, 6), (1 << 63) - 1, np.int64)
+    assert _create(lib, demand=top, recompute=top) == lib.PP_EOVERFLOW
+    W, n = 16, 4096
+    base = dict(n=n, W=W, parent=np.full(n, -1, np.int32), weight=np.ones(n, np.int32),
+                demand=np.ones((W, n), np.int64), recompute=np.ones((W, n), np.int64),
+                transfer=np.ones((W, W, n), np.int64), mode=1, budget=np.full(W, 8, np.int32))
+    tr = base["transfer"].copy()
+    tr[W - 1, W - 2, n - 3] = -5                     # in the last thread's slice
+    assert _create(lib, **{**base, "transfer": tr}) == lib.PP_EINVAL
+    assert "transfer" in lib.last_error()
+    dem = base["demand"].copy()
+    dem[W // 2, n // 2] = -1
+    assert _create(lib, **{**base, "demand": dem}) == lib.PP_EINVAL
+    assert "demand" in lib.last_error()
+    # every slice's partial sum is below 2^62, their total above
+    spread = np.full((W, n), (1 << 62) // (W * n // 2), np.int64)
+    assert _create(lib, **{**base, "demand": spread, "recompute": np.zeros((W, n), np.int64)}) == lib.PP_EOVERFLOW
+    assert "sum of demand" in lib.last_error()
+
+
 def test_row_plan_preorder_matches_definition(lib):
     """The library's preorder (independent of the oracle's) follows Section IV-A."""
     rng = np.random.default_rng(2)
