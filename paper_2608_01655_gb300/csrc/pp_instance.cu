@@ -258,87 +258,11 @@ static pp_status upload(T **dst, const T *src, size_t count, cudaStream_t st)
     return PP_OK;
 }
 
-static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
-                             const int64_t *demand, const int64_t *recompute,
-                             const int64_t *transfer, int32_t mode, const int32_t *budget,
-                             cudaStream_t st, pp_instance *inst)
+// The tree's host tables of an instance: preorder, next, weights by
+// position, the traceback's skip depth, the skip-row stack plan, budgets.
+static pp_status build_host_tables(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
+                                   int32_t mode, const int32_t *budget, pp_instance *inst)
 {
-    if (n < 0) return fail(PP_EINVAL, "n must be >= 0");
-    if (W < 1 || W > 32) return fail(PP_EINVAL, "W must be in 1..32");
-    if (mode != PP_TRANSFER_REQUESTER && mode != PP_TRANSFER_SOURCE)
-        return fail(PP_EINVAL, "transfer_mode must be 0 (requester) or 1 (source)");
-    if (!budget || (n > 0 && (!parent || !weight || !demand || !recompute || !transfer)))
-        return fail(PP_EINVAL, "null input pointer");
-    for (int32_t m = 0; m < W; ++m)
-        if (budget[m] < 0) return fail(PP_EINVAL, "budget must be >= 0");
-    for (int32_t v = 0; v < n; ++v) {
-        if (parent[v] < -1 || parent[v] >= n || parent[v] == v)
-            return fail(PP_ENOTTREE, "parent id out of range or self-parent at node " + std::to_string(v));
-        if (weight[v] < 1) return fail(PP_EINVAL, "chunk weight must be >= 1");
-    }
-    const size_t Wn = (size_t)W * n;
-    const size_t tn = mode == PP_TRANSFER_SOURCE ? (size_t)W * Wn : Wn;
-    // Three exact sums bound every int64 value the library forms:
-    //  sum Lambda * w: objectives (Eq. 4, Eq. 6), marginals and DP values;
-    //  sum Lambda:     the Popularity safeguard's DP values (profit Lambda);
-    //  sum w:          the epoch update's one-time cost (at most one w per (m, b)).
-    // The cost arrays are checked before anything is allocated, on up to 16
-    // host threads when they are large (the source-dependent transfer costs
-    // are W^2 n values: 102 MB at the paper-scale workload).
-    // Unsigned 128-bit sums (a negative value sets bit 63 of the OR and fails
-    // before its sum is used); the products and the running sum of products
-    // are capped at 2^63, above the 2^62 limit, so nothing wraps.
-    using u128 = unsigned __int128;
-    const u128 cap = (u128)1 << 63;
-    struct Part {
-        u128 total = 0, demand = 0, recompute = 0;
-        uint64_t dr_bits = 0, t_bits = 0;          // OR of the values: bit 63 = a negative one
-    };
-    const size_t work = Wn + tn;
-    const unsigned hw = std::max(1u, std::thread::hardware_concurrency());
-    const int nth = work < ((size_t)1 << 20) ? 1 : (int)std::min<unsigned>(hw, 16);
-    std::vector<Part> parts(nth);
-    auto check = [&](int q) {
-        Part &P = parts[q];
-        const size_t a = Wn * q / nth, b = Wn * (q + 1) / nth;
-        for (size_t x = a; x < b; ++x) {
-            const uint64_t dv = (uint64_t)demand[x], rv = (uint64_t)recompute[x];
-            P.dr_bits |= dv | rv;
-            const u128 pr = (u128)dv * rv;
-            P.total = std::min<u128>(P.total + std::min(pr, cap), cap);
-            P.demand += dv;
-            P.recompute += rv;
-        }
-        const size_t c = tn * q / nth, d = tn * (q + 1) / nth;
-        uint64_t tb = 0;
-        for (size_t x = c; x < d; ++x) tb |= (uint64_t)transfer[x];
-        P.t_bits = tb;
-    };
-    if (nth == 1) {
-        check(0);
-    } else {
-        std::vector<std::thread> pool;
-        pool.reserve(nth - 1);
-        for (int q = 1; q < nth; ++q) pool.emplace_back(check, q);
-        check(0);
-        for (auto &th : pool) th.join();
-    }
-    u128 total = 0, sum_demand = 0, sum_recompute = 0;
-    uint64_t dr_bits = 0, t_bits = 0;
-    for (const Part &P : parts) {
-        total = std::min<u128>(total + P.total, cap);
-        sum_demand += P.demand;
-        sum_recompute += P.recompute;
-        dr_bits |= P.dr_bits;
-        t_bits |= P.t_bits;
-    }
-    if (dr_bits >> 63) return fail(PP_EINVAL, "negative demand or recompute cost");
-    if (t_bits >> 63) return fail(PP_EINVAL, "negative transfer cost");
-    const u128 lim = (u128)1 << 62;
-    if (total > lim) return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
-    if (sum_demand > lim) return fail(PP_EOVERFLOW, "sum of demand exceeds 2^62");
-    if (sum_recompute > lim) return fail(PP_EOVERFLOW, "sum of recompute costs exceeds 2^62");
-
     inst->n = n;
     inst->W = W;
     inst->mode = mode;
@@ -369,6 +293,91 @@ static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const 
     if (!build_row_meta(n, inst->h_next, inst->h_meta, &inst->stack_depth, &inst->h_wpre, &inst->h_wave))
         return fail(PP_EINVAL, "skip-row stack deeper than supported");
     inst->h_budget.assign(budget, budget + W);
+    return PP_OK;
+}
+
+static pp_status create_impl(int32_t n, int32_t W, const int32_t *parent, const int32_t *weight,
+                             const int64_t *demand, const int64_t *recompute,
+                             const int64_t *transfer, int32_t mode, const int32_t *budget,
+                             cudaStream_t st, pp_instance *inst)
+{
+    if (n < 0) return fail(PP_EINVAL, "n must be >= 0");
+    if (W < 1 || W > 32) return fail(PP_EINVAL, "W must be in 1..32");
+    if (mode != PP_TRANSFER_REQUESTER && mode != PP_TRANSFER_SOURCE)
+        return fail(PP_EINVAL, "transfer_mode must be 0 (requester) or 1 (source)");
+    if (!budget || (n > 0 && (!parent || !weight || !demand || !recompute || !transfer)))
+        return fail(PP_EINVAL, "null input pointer");
+    for (int32_t m = 0; m < W; ++m)
+        if (budget[m] < 0) return fail(PP_EINVAL, "budget must be >= 0");
+    for (int32_t v = 0; v < n; ++v) {
+        if (parent[v] < -1 || parent[v] >= n || parent[v] == v)
+            return fail(PP_ENOTTREE, "parent id out of range or self-parent at node " + std::to_string(v));
+        if (weight[v] < 1) return fail(PP_EINVAL, "chunk weight must be >= 1");
+    }
+    const size_t Wn = (size_t)W * n;
+    const size_t tn = mode == PP_TRANSFER_SOURCE ? (size_t)W * Wn : Wn;
+    // Three exact sums bound every int64 value the library forms:
+    //  sum Lambda * w: objectives (Eq. 4, Eq. 6), marginals and DP values;
+    //  sum Lambda:     the Popularity safeguard's DP values (profit Lambda);
+    //  sum w:          the epoch update's one-time cost (at most one w per (m, b)).
+    // The cost arrays are checked before anything is allocated, on up to 16
+    // host threads when they are large (the source-dependent transfer costs
+    // are W^2 n values: 102 MB at the paper-scale workload), while this thread
+    // builds the tree's host tables; cost errors are reported first.
+    // Unsigned 128-bit sums (a negative value sets bit 63 of the OR and fails
+    // before its sum is used); the products and the running sum of products
+    // are capped at 2^63, above the 2^62 limit, so nothing wraps.
+    using u128 = unsigned __int128;
+    const u128 cap = (u128)1 << 63;
+    struct Part {
+        u128 total = 0, demand = 0, recompute = 0;
+        uint64_t dr_bits = 0, t_bits = 0;          // OR of the values: bit 63 = a negative one
+    };
+    const size_t work = Wn + tn;
+    const unsigned hw = std::max(1u, std::thread::hardware_concurrency());
+    const int nth = work < ((size_t)1 << 20) ? 1 : (int)std::min<unsigned>(hw, 16);
+    std::vector<Part> parts(nth);
+    auto check = [&](int q) {
+        Part &P = parts[q];
+        const size_t a = Wn * q / nth, b = Wn * (q + 1) / nth;
+        for (size_t x = a; x < b; ++x) {
+            const uint64_t dv = (uint64_t)demand[x], rv = (uint64_t)recompute[x];
+            P.dr_bits |= dv | rv;
+            const u128 pr = (u128)dv * rv;
+            P.total = std::min<u128>(P.total + std::min(pr, cap), cap);
+            P.demand += dv;
+            P.recompute += rv;
+        }
+        const size_t c = tn * q / nth, d = tn * (q + 1) / nth;
+        uint64_t tb = 0;
+        for (size_t x = c; x < d; ++x) tb |= (uint64_t)transfer[x];
+        P.t_bits = tb;
+    };
+    std::vector<std::thread> pool;
+    if (nth == 1) {
+        check(0);
+    } else {
+        pool.reserve(nth);
+        for (int q = 0; q < nth; ++q) pool.emplace_back(check, q);
+    }
+    const pp_status tables = build_host_tables(n, W, parent, weight, mode, budget, inst);
+    for (auto &th : pool) th.join();
+    u128 total = 0, sum_demand = 0, sum_recompute = 0;
+    uint64_t dr_bits = 0, t_bits = 0;
+    for (const Part &P : parts) {
+        total = std::min<u128>(total + P.total, cap);
+        sum_demand += P.demand;
+        sum_recompute += P.recompute;
+        dr_bits |= P.dr_bits;
+        t_bits |= P.t_bits;
+    }
+    if (dr_bits >> 63) return fail(PP_EINVAL, "negative demand or recompute cost");
+    if (t_bits >> 63) return fail(PP_EINVAL, "negative transfer cost");
+    const u128 lim = (u128)1 << 62;
+    if (total > lim) return fail(PP_EOVERFLOW, "sum of demand * recompute exceeds 2^62");
+    if (sum_demand > lim) return fail(PP_EOVERFLOW, "sum of demand exceeds 2^62");
+    if (sum_recompute > lim) return fail(PP_EOVERFLOW, "sum of recompute costs exceeds 2^62");
+    if (tables != PP_OK) return tables;
 
     PP_CUDA(cudaGetDevice(&inst->device));
     PP_CUDA(cudaDeviceGetAttribute(&inst->sm_count, cudaDevAttrMultiProcessorCount, inst->device));

@@ -109,6 +109,13 @@ def test_create_validation_large_and_extreme(lib):
     dem[W // 2, n // 2] = -1
     assert _create(lib, **{**base, "demand": dem}) == lib.PP_EINVAL
     assert "demand" in lib.last_error()
+    # the tree's tables are built while the costs are checked: a cost error
+    # is still the one reported when the tree is bad as well
+    cyc = base["parent"].copy()
+    cyc[:3] = [1, 2, 0]
+    assert _create(lib, **{**base, "parent": cyc}) == lib.PP_ENOTTREE
+    assert _create(lib, **{**base, "parent": cyc, "demand": dem}) == lib.PP_EINVAL
+    assert "demand" in lib.last_error()
     # every slice's partial sum is below 2^62, their total above
     spread = np.full((W, n), (1 << 62) // (W * n // 2), np.int64)
     assert _create(lib, **{**base, "demand": spread, "recompute": np.zeros((W, n), np.int64)}) == lib.PP_EOVERFLOW
